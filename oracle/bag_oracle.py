@@ -1,0 +1,457 @@
+"""fp64 CPU oracle for BAG's cached DiT sampling path.
+
+TEST INFRASTRUCTURE ONLY.  This module is imported by the tests, by the package's smoke
+check and by the benchmark's CPU-baseline leg; the product path never calls it.  It
+shares no code with the CUDA library: only the seeded input generator (synth.py, which
+holds none of the method's arithmetic) feeds both.
+
+What it computes, and from which passage:
+  * Budget-exact inference, Algorithm 2 and Sec. 3.2 "Budget-exact inference":
+    m_0 = 1 with c = 1; for t >= 1 the gate decides m_t = [sigma(z_t) > tau], then
+    "B - c >= T - t => m_t = 1", then "B - c = 0 => m_t = 0"; a full step runs the
+    network and refreshes the cache (c += 1), any other step reuses the cached residual.
+  * The problem setup of Sec. 3.1: binary mask m with ||m||_1 = B, m_0 = 1; a reused
+    step goes "through the standard residual path" (plain residual reuse, Sec. 2).
+  * The gate z_t = g_theta(s_bud, s_traj) of Eq. 1, in the 3-input form the build
+    targets (remaining-budget fraction, remaining-steps fraction, drift signal) with
+    all six scalars of Eq. 3 logged beside it.
+  * The trajectory signal: relative L1 change of the first block's modulated input
+    against the last fully computed step (the drift entry of Eq. 3 with the L1 norm).
+  * The DiT network evaluated at full steps: adaLN-modulated MMDiT blocks (modulated
+    LayerNorm, QKV projection with RoPE, joint attention, output projection, GELU MLP,
+    gated residuals).  The paper names the backbones (FLUX.1-dev, Qwen-Image, Wan2.1;
+    Sec. 4.1) but not their internals; the block conventions below are the public ones.
+  * A flow-matching Euler sampler over sigma_i = 1 - i / T (Sec. 3.1 "T denoising
+    steps"; flow matching cited in Sec. 1).
+
+Readings where the paper is silent (also listed in the design notes):
+  LayerNorm without affine, eps 1e-6; modulation (1 + scale) * LN(x) + shift; GELU with
+  the tanh approximation; attention scale 1/sqrt(head_dim); joint sequence order
+  [text; image]; RoPE on interleaved pairs, theta = 10000, per-axis frequencies
+  theta^(-2j/d_axis), text tokens at position 0; timestep embedding cos-then-sin of
+  1000 * sigma_t over 128 frequencies exp(-ln(10000) j / 128); gate hidden activation
+  ReLU; decision on z > logit(tau) (z = logit(tau) reuses); cached residual R = image
+  stream after the last block minus the image stream entering the first block;
+  text stream not advanced on reused steps.
+
+Precision: everything in float64 except the gate, which is evaluated in float32 in a
+fixed operation order (each product and sum rounded separately) because its output is a
+binary decision that both implementations must take in the same precision.
+
+Parity pins: see tests/test_oracle_pins.py.  Every function below is pinned by at least
+one closed form, invariant, special case or brute-force check there.
+"""
+
+import math
+
+import numpy as np
+
+TEMB_DIM = 256
+ROPE_THETA = 10000.0
+LN_EPS = 1e-6
+
+
+# ---------------------------------------------------------------------------
+# elementwise pieces
+# ---------------------------------------------------------------------------
+def silu(x):
+    return x / (1.0 + np.exp(-x))
+
+
+def gelu_tanh(x):
+    """GELU, tanh approximation (public FLUX/Wan convention; the paper is silent)."""
+    return 0.5 * x * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (x + 0.044715 * x ** 3)))
+
+
+def layer_norm(x, eps=LN_EPS):
+    """Row-wise LayerNorm without affine parameters."""
+    mu = x.mean(axis=-1, keepdims=True)
+    var = ((x - mu) ** 2).mean(axis=-1, keepdims=True)
+    return (x - mu) / np.sqrt(var + eps)
+
+
+def modulate(xn, shift, scale):
+    """adaLN modulation (1 + scale) * xn + shift."""
+    return xn * (1.0 + scale) + shift
+
+
+def linear(x, w, b=None):
+    """y = x W^T + b with W stored [out, in]."""
+    y = x @ w.T
+    if b is not None:
+        y = y + b
+    return y
+
+
+def timestep_embedding(tval, dim=TEMB_DIM):
+    """Sinusoidal embedding of a scalar timestep: [cos(t f_j), sin(t f_j)], j < dim/2."""
+    half = dim // 2
+    freqs = np.exp(-math.log(10000.0) * np.arange(half, dtype=np.float64) / half)
+    args = float(tval) * freqs
+    return np.concatenate([np.cos(args), np.sin(args)])
+
+
+def sigma_grid(T):
+    """Flow-matching noise levels sigma_i = 1 - i/T, i = 0..T (no shift)."""
+    return 1.0 - np.arange(T + 1, dtype=np.float64) / T
+
+
+# ---------------------------------------------------------------------------
+# rotary embedding and attention
+# ---------------------------------------------------------------------------
+def token_positions(cfg):
+    """(frame, row, col) of each joint-sequence token: text first at 0, image row-major."""
+    f, r, c = cfg["grid"]
+    img = np.array([(a, b, e) for a in range(f) for b in range(r) for e in range(c)],
+                   dtype=np.float64).reshape(-1, 3)
+    if cfg["kind"] == "wan":
+        return img
+    return np.concatenate([np.zeros((cfg["n_txt"], 3)), img], axis=0)
+
+
+def rope_angles(pos, axes, theta=ROPE_THETA):
+    """Rotation angle of every (token, pair): pairs are laid out axis after axis; pair j
+    of an axis of width d_a turns by pos_a * theta^(-2j/d_a)."""
+    cols = []
+    for a, da in enumerate(axes):
+        if da == 0:
+            continue
+        j = np.arange(da // 2, dtype=np.float64)
+        omega = theta ** (-2.0 * j / da)
+        cols.append(pos[:, a:a + 1] * omega[None, :])
+    return np.concatenate(cols, axis=1)
+
+
+def apply_rope(x, ang):
+    """Rotate interleaved pairs (x[2j], x[2j+1]) of x [N, H, Dh] by ang [N, Dh/2]."""
+    c = np.cos(ang)[:, None, :]
+    s = np.sin(ang)[:, None, :]
+    x0, x1 = x[..., 0::2], x[..., 1::2]
+    out = np.empty_like(x)
+    out[..., 0::2] = x0 * c - x1 * s
+    out[..., 1::2] = x0 * s + x1 * c
+    return out
+
+
+def softmax_rows(s):
+    m = s.max(axis=-1, keepdims=True)
+    e = np.exp(s - m)
+    return e / e.sum(axis=-1, keepdims=True)
+
+
+def attention(q, k, v, q_rows=None):
+    """softmax(q k^T / sqrt(Dh)) v per head.  q [Nq, H, Dh], k, v [Nk, H, Dh].
+
+    q_rows optionally restricts the query rows (the result then has len(q_rows) rows)."""
+    if q_rows is not None:
+        q = q[q_rows]
+    dh = q.shape[-1]
+    out = np.empty(q.shape, dtype=np.float64)
+    for h in range(q.shape[1]):
+        p = softmax_rows(q[:, h, :] @ k[:, h, :].T / math.sqrt(dh))
+        out[:, h, :] = p @ v[:, h, :]
+    return out
+
+
+# ---------------------------------------------------------------------------
+# blocks
+# ---------------------------------------------------------------------------
+def _heads(x, H):
+    return x.reshape(x.shape[0], H, -1)
+
+
+def single_block(h, mod, W, ang, H, rows=None):
+    """Single-stream block on the joint sequence h [N, d]; mod = (shift, scale, gate).
+
+    LN-mod -> linear1 (d -> 3d + F: q, k, v, mlp) -> RoPE(q, k) -> attention;
+    GELU(mlp); linear2 on [attn | GELU(mlp)] -> gated residual.
+    rows: compute the output only at these rows (the others are not returned)."""
+    d = h.shape[1]
+    shift, scale, gate = mod[:d], mod[d:2 * d], mod[2 * d:3 * d]
+    xn = modulate(layer_norm(h), shift, scale)
+    w1, b1 = W["lin1_w"], W["lin1_b"]
+    qkv = linear(xn, w1[:3 * d], b1[:3 * d])
+    q = apply_rope(_heads(qkv[:, :d], H), ang)
+    k = apply_rope(_heads(qkv[:, d:2 * d], H), ang)
+    v = _heads(qkv[:, 2 * d:], H)
+    sel = slice(None) if rows is None else rows
+    a = attention(q, k, v, q_rows=rows).reshape(-1, d)
+    mlp = gelu_tanh(linear(xn[sel], w1[3 * d:], b1[3 * d:]))
+    o = linear(np.concatenate([a, mlp], axis=1), W["lin2_w"], W["lin2_b"])
+    return h[sel] + gate * o
+
+
+def _mlp(x, wu, bu, wd, bd):
+    return linear(gelu_tanh(linear(x, wu, bu)), wd, bd)
+
+
+def double_block(img, txt, mod_img, mod_txt, W, ang, H):
+    """Double-stream (MMDiT) block: separate weights per stream, joint attention over
+    [txt; img].  mod_* = (shift1, scale1, gate1, shift2, scale2, gate2)."""
+    d = img.shape[1]
+    nx = txt.shape[0]
+
+    def chunks(m):
+        return [m[i * d:(i + 1) * d] for i in range(6)]
+
+    mi, mt = chunks(mod_img), chunks(mod_txt)
+    qkv_i = linear(modulate(layer_norm(img), mi[0], mi[1]), W["img_qkv_w"], W["img_qkv_b"])
+    qkv_t = linear(modulate(layer_norm(txt), mt[0], mt[1]), W["txt_qkv_w"], W["txt_qkv_b"])
+    qkv = np.concatenate([qkv_t, qkv_i], axis=0)
+    q = apply_rope(_heads(qkv[:, :d], H), ang)
+    k = apply_rope(_heads(qkv[:, d:2 * d], H), ang)
+    v = _heads(qkv[:, 2 * d:], H)
+    a = attention(q, k, v).reshape(-1, d)
+    a_t, a_i = a[:nx], a[nx:]
+    img = img + mi[2] * linear(a_i, W["img_proj_w"], W["img_proj_b"])
+    txt = txt + mt[2] * linear(a_t, W["txt_proj_w"], W["txt_proj_b"])
+    img = img + mi[5] * _mlp(modulate(layer_norm(img), mi[3], mi[4]),
+                             W["img_up_w"], W["img_up_b"], W["img_down_w"], W["img_down_b"])
+    txt = txt + mt[5] * _mlp(modulate(layer_norm(txt), mt[3], mt[4]),
+                             W["txt_up_w"], W["txt_up_b"], W["txt_down_w"], W["txt_down_b"])
+    return img, txt
+
+
+def wan_block(x, ctx, e, W, ang, H):
+    """Wan-style block: modulated self-attention with 3D RoPE, cross-attention to the
+    text context (plain LayerNorm on the query side, no gate), modulated GELU FFN.
+    e = (shift1, scale1, gate1, shift2, scale2, gate2)."""
+    d = x.shape[1]
+    ch = [e[i * d:(i + 1) * d] for i in range(6)]
+    qkv = linear(modulate(layer_norm(x), ch[0], ch[1]), W["sa_qkv_w"], W["sa_qkv_b"])
+    q = apply_rope(_heads(qkv[:, :d], H), ang)
+    k = apply_rope(_heads(qkv[:, d:2 * d], H), ang)
+    v = _heads(qkv[:, 2 * d:], H)
+    x = x + ch[2] * linear(attention(q, k, v).reshape(-1, d), W["sa_o_w"], W["sa_o_b"])
+    qc = _heads(linear(layer_norm(x), W["ca_q_w"], W["ca_q_b"]), H)
+    kv = linear(ctx, W["ca_kv_w"], W["ca_kv_b"])
+    kc, vc = _heads(kv[:, :d], H), _heads(kv[:, d:], H)
+    x = x + linear(attention(qc, kc, vc).reshape(-1, d), W["ca_o_w"], W["ca_o_b"])
+    x = x + ch[5] * _mlp(modulate(layer_norm(x), ch[3], ch[4]),
+                         W["ffn_up_w"], W["ffn_up_b"], W["ffn_down_w"], W["ffn_down_b"])
+    return x
+
+
+# ---------------------------------------------------------------------------
+# network pieces around the stack
+# ---------------------------------------------------------------------------
+def conditioning(cfg, G, sigma, pooled):
+    """vec = MLP(sinusoid(1000 sigma)) (+ pooled text vector except for Wan)."""
+    e = timestep_embedding(1000.0 * sigma)
+    temb = linear(silu(linear(e, G["t1_w"], G["t1_b"])), G["t2_w"], G["t2_b"])
+    if cfg["kind"] == "wan":
+        return temb
+    return temb + pooled
+
+
+def block_modulation(cfg, G, blk, vec):
+    """Per-block modulation vectors from the conditioning vector."""
+    if blk["type"] == "single":
+        return linear(silu(vec), blk["mod_w"], blk["mod_b"])
+    if blk["type"] == "double":
+        return (linear(silu(vec), blk["img_mod_w"], blk["img_mod_b"]),
+                linear(silu(vec), blk["txt_mod_w"], blk["txt_mod_b"]))
+    # Wan: one shared projection of the time embedding plus a per-block table
+    return linear(silu(vec), G["tproj_w"], G["tproj_b"]) + blk["mod_tab"]
+
+
+def first_modulated_input(cfg, G, blocks, vec, h_img):
+    """Image-stream input of the first block after its first LN-modulation: the
+    observable the trajectory signal reads."""
+    d = cfg["hidden"]
+    mod = block_modulation(cfg, G, blocks[0], vec)
+    if blocks[0]["type"] == "double":
+        mod = mod[0]
+    return modulate(layer_norm(h_img), mod[:d], mod[d:2 * d])
+
+
+def patch_embed(G, x):
+    return linear(x, G["pe_w"], G["pe_b"])
+
+
+def run_stack(cfg, G, blocks, vec, h_img, txt):
+    """Full network stack on the image stream h_img [N_i, d] with text txt; returns the
+    image stream after the last block."""
+    H = cfg["heads"]
+    pos = token_positions(cfg)
+    ang = rope_angles(pos, cfg["rope_axes"])
+    if cfg["kind"] == "wan":
+        x = h_img
+        for blk in blocks:
+            x = wan_block(x, txt, block_modulation(cfg, G, blk, vec), blk, ang, H)
+        return x
+    img, tx = h_img, txt
+    nx = txt.shape[0]
+    singles_started = False
+    hj = None
+    for blk in blocks:
+        mod = block_modulation(cfg, G, blk, vec)
+        if blk["type"] == "double":
+            assert not singles_started
+            img, tx = double_block(img, tx, mod[0], mod[1], blk, ang, H)
+        else:
+            if not singles_started:
+                hj = np.concatenate([tx, img], axis=0)
+                singles_started = True
+            hj = single_block(hj, mod, blk, ang, H)
+    if singles_started:
+        img = hj[nx:]
+    return img
+
+
+def final_layer(G, vec, h_img):
+    d = h_img.shape[1]
+    mod = linear(silu(vec), G["fmod_w"], G["fmod_b"])
+    return linear(modulate(layer_norm(h_img), mod[:d], mod[d:]), G["fin_w"], G["fin_b"])
+
+
+def rel_l1(a, b):
+    """Relative L1 change sum|a - b| / sum|b| (the drift entry of Eq. 3, L1 norm)."""
+    return float(np.abs(a - b).sum() / np.abs(b).sum())
+
+
+# ---------------------------------------------------------------------------
+# gate and pacing (Eq. 1, Eq. 3, Algorithm 2)
+# ---------------------------------------------------------------------------
+F32 = np.float32
+
+
+def gate_threshold(tau):
+    """Decision threshold on the logit: sigma(z) > tau  <=>  z > log(tau / (1 - tau))."""
+    return F32(math.log(tau / (1.0 - tau)))
+
+
+def gate_features(B, T, c, t, drift):
+    """The three gate inputs at step t with c evaluations already spent: remaining-budget
+    fraction (B - c)/B (Eq. 3), remaining-steps fraction (T - t)/T, drift signal."""
+    return [F32(B - c) / F32(B), F32(T - t) / F32(T), F32(drift)]
+
+
+def gate_logit(f, g):
+    """z = w2 . ReLU(W1 ((f - mu) / sd) + b1) + b2 in float32, fixed order: every product
+    and every sum rounded on its own, inputs visited in index order."""
+    fz = [(F32(f[i]) - F32(g["mu"][i])) / F32(g["sd"][i]) for i in range(len(f))]
+    w1, b1, w2, b2 = g["w1"], g["b1"], g["w2"], g["b2"]
+    z = F32(b2[0])
+    for j in range(w1.shape[0]):
+        hj = F32(b1[j])
+        for i in range(len(fz)):
+            hj = F32(hj + F32(F32(w1[j, i]) * fz[i]))
+        if not hj > F32(0.0):
+            hj = F32(0.0)
+        z = F32(z + F32(F32(w2[j]) * hj))
+    return z
+
+
+def pace(gate_bit, B, T, c, t):
+    """Algorithm 2's forced rules applied to the gate's bit at step t >= 1."""
+    m = 1 if gate_bit else 0
+    if B - c >= T - t:
+        m = 1        # spend the remainder
+    if B - c == 0:
+        m = 0        # budget exhausted
+    return m
+
+
+def schedule_from_gate_bits(bits, B, T):
+    """Mask produced by Algorithm 2 from a sequence of raw gate bits (bits[0] unused)."""
+    m = [1]
+    c = 1
+    for t in range(1, T):
+        mt = pace(bits[t], B, T, c, t)
+        m.append(mt)
+        c += mt
+    return m
+
+
+# ---------------------------------------------------------------------------
+# the sampler (Algorithm 2 with the network, the signal and the residual cache)
+# ---------------------------------------------------------------------------
+def to64(W):
+    """Upcast a weight tree (as produced by the seeded generator) to float64."""
+    out = {"global": {k: np.asarray(v, np.float64) for k, v in W["global"].items()},
+           "blocks": []}
+    for blk in W["blocks"]:
+        out["blocks"].append(None if blk is None else
+                             {k: (v if k == "type" else np.asarray(v, np.float64))
+                              for k, v in blk.items()})
+    return out
+
+
+def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=None):
+    """One sample of T Euler steps under Algorithm 2.
+
+    policy         'bag' (gate + pacing), 'full' (uncached: every step computes), or a
+                   list of T mask bits to follow (a static schedule).
+    drift_override optional per-step drift values (index t) to feed the gate instead of
+                   the oracle's own; used to take the decision on another
+                   implementation's logged gate inputs.
+    Returns dict(x=final latent, mask, log=[per-step dict]).
+    """
+    if not (1 <= B <= T):
+        raise ValueError("need 1 <= B <= T")
+    W = to64(W)
+    G, blocks = W["global"], W["blocks"]
+    x = np.asarray(inputs["x"], np.float64)
+    txt = np.asarray(inputs["txt"], np.float64)
+    pooled = np.asarray(inputs["pooled"], np.float64)
+    sig = sigma_grid(T)
+    thr = gate_threshold(tau)
+    c = 0
+    t_last = -1
+    R = m_last = m_prev = None
+    mask, log = [], []
+    for t in range(T):
+        vec = conditioning(cfg, G, sig[t], pooled)
+        h_in = patch_embed(G, x)
+        m_t = first_modulated_input(cfg, G, blocks, vec, h_in)
+        rec = {"t": t, "c_before": c}
+        if t == 0:
+            full = 1
+        else:
+            drift = rel_l1(m_t, m_last)
+            rec["drift"] = drift
+            # the six scalars of Eq. 3, logged
+            rec["s_bud"] = [B / T, (B - c) / B, (B - c) / (T - t)]
+            rec["s_traj"] = [t - t_last, drift, rel_l1(m_t, m_prev)]
+            used = drift if drift_override is None else drift_override[t]
+            f = gate_features(B, T, c, t, used)
+            z = gate_logit(f, gate)
+            rec["features"] = [float(v) for v in f]
+            rec["z"] = float(z)
+            gbit = 1 if z > thr else 0
+            if policy == "bag":
+                full = pace(gbit, B, T, c, t)
+            elif policy == "full":
+                full = 1
+            else:
+                full = int(policy[t])
+        rec["full"] = full
+        if full:
+            h_out = run_stack(cfg, G, blocks, vec, h_in, txt)
+            R = h_out - h_in
+            m_last = m_t
+            t_last = t
+            c += 1
+        else:
+            h_out = h_in + R
+        m_prev = m_t
+        v = final_layer(G, vec, h_out)
+        x = x + (sig[t + 1] - sig[t]) * v
+        mask.append(full)
+        log.append(rec)
+    return {"x": x, "mask": mask, "log": log, "nfe": c}
+
+
+def forward_block(cfg, W, block_index, h_joint, vec, rows=None):
+    """One block of the stack applied to a given joint stream (text rows first for the
+    MMDiT kinds; image rows only for Wan, with txt the context).  Used to check a single
+    block at full width on sampled rows."""
+    W = to64(W)
+    G, blk = W["global"], W["blocks"][block_index]
+    H = cfg["heads"]
+    ang = rope_angles(token_positions(cfg), cfg["rope_axes"])
+    mod = block_modulation(cfg, G, blk, vec)
+    if blk["type"] == "single":
+        return single_block(h_joint, mod, blk, ang, H, rows=rows)
+    raise NotImplementedError(blk["type"])

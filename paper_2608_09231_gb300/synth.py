@@ -1,0 +1,228 @@
+"""Seeded synthetic inputs: one counter-based generator, host side (numpy).
+
+This module holds none of the method's arithmetic.  It only turns (seed, tensor key,
+element index) into numbers, so that the fp64 oracle and the CUDA path see the same
+weights and inputs.  The CUDA library carries its own implementation of the same
+generator (device kernel for the large weight tensors, host C++ for the gate); both are
+written from the published definition of SplitMix64 (Steele, Lea and Flood, "Fast
+splittable pseudorandom number generators", OOPSLA 2014):
+
+    state_i = s + (i + 1) * 0x9E3779B97F4A7C15          (mod 2^64)
+    out_i   = mix(state_i)
+    mix(z)  : z ^= z >> 30; z *= 0xBF58476D1CE4E5B9;
+              z ^= z >> 27; z *= 0x94D049BB133111EB; z ^= z >> 31
+
+with the stream start  s = mix(seed * 0x9E3779B97F4A7C15 ^ mix(key)).
+
+Distributions (all exactly reproducible in IEEE fp32 on any machine):
+  normal(std)   Irwin-Hall sum of the four 16-bit chunks of out_i, centred:
+                q = a+b+c+d - 131070 (an integer, exact in fp32), value = fp32(q) * c32
+                with c32 = fp32(std * sqrt(3) / 65536), so the variance is std^2.
+  uniform(lo,hi) u = fp32(out_i >> 40) * 2^-24; value = lo + (hi - lo) * u, each
+                operation rounded separately in fp32.
+bf16 storage uses round-to-nearest-even of the fp32 value.
+"""
+
+import numpy as np
+
+from .configs import TEMB_DIM
+
+GOLDEN = np.uint64(0x9E3779B97F4A7C15)
+M1 = np.uint64(0xBF58476D1CE4E5B9)
+M2 = np.uint64(0x94D049BB133111EB)
+
+
+def _mix(z):
+    z = np.asarray(z, dtype=np.uint64)
+    with np.errstate(over="ignore"):
+        z = (z ^ (z >> np.uint64(30))) * M1
+        z = (z ^ (z >> np.uint64(27))) * M2
+    return z ^ (z >> np.uint64(31))
+
+
+def stream_start(seed, key):
+    with np.errstate(over="ignore"):
+        a = np.uint64(seed) * GOLDEN
+    return _mix(a ^ _mix(np.uint64(key)))
+
+
+def raw_u64(seed, key, n, offset=0):
+    s = stream_start(seed, key)
+    idx = np.arange(offset + 1, offset + n + 1, dtype=np.uint64)
+    with np.errstate(over="ignore"):
+        st = s + idx * GOLDEN
+    return _mix(st)
+
+
+def normal_scale(std):
+    return np.float32(float(std) * np.sqrt(3.0) / 65536.0)
+
+
+def normal(seed, key, n, std, offset=0, chunk=1 << 24):
+    """n fp32 samples of the Irwin-Hall(4) normal approximation with the given std."""
+    out = np.empty(n, dtype=np.float32)
+    c32 = normal_scale(std)
+    mask = np.uint64(0xFFFF)
+    for lo in range(0, n, chunk):
+        m = min(chunk, n - lo)
+        u = raw_u64(seed, key, m, offset + lo)
+        q = ((u & mask) + ((u >> np.uint64(16)) & mask) + ((u >> np.uint64(32)) & mask)
+             + (u >> np.uint64(48))).astype(np.int64) - 131070
+        out[lo:lo + m] = q.astype(np.float32) * c32
+    return out
+
+
+def uniform(seed, key, n, lo, hi):
+    u = raw_u64(seed, key, n)
+    f = (u >> np.uint64(40)).astype(np.float32) * np.float32(2.0 ** -24)
+    return np.float32(lo) + (np.float32(hi) - np.float32(lo)) * f
+
+
+def bf16_round(x):
+    """Round fp32 values to the nearest bf16 (ties to even); returns fp32 values."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    u = x.view(np.uint32).astype(np.uint64)
+    u = (u + np.uint64(0x7FFF) + ((u >> np.uint64(16)) & np.uint64(1))) & np.uint64(0xFFFF0000)
+    return u.astype(np.uint32).view(np.float32).reshape(x.shape)
+
+
+def bf16_bits(x):
+    """Bit pattern (uint16) of fp32 values that are already bf16-representable."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    return (x.view(np.uint32) >> np.uint32(16)).astype(np.uint16)
+
+
+# ---------------------------------------------------------------------------
+# Tensor inventory.  key = block_slot * 256 + tensor_id; block_slot 0 holds the global
+# tensors, slot 1 + i the i-th block in execution order (double blocks, then single).
+# Weights are [out, in] row-major (out features x in features).
+# ---------------------------------------------------------------------------
+WEIGHT_STD = 0.02
+BIAS_STD = 0.02
+
+GLOBAL_IDS = {
+    "pe_w": 0, "pe_b": 1, "t1_w": 2, "t1_b": 3, "t2_w": 4, "t2_b": 5,
+    "fmod_w": 6, "fmod_b": 7, "fin_w": 8, "fin_b": 9, "tproj_w": 10, "tproj_b": 11,
+}
+SINGLE_IDS = {"mod_w": 0, "mod_b": 1, "lin1_w": 2, "lin1_b": 3, "lin2_w": 4, "lin2_b": 5}
+DOUBLE_IDS = {}
+for _i, _s in enumerate(("img", "txt")):
+    for _j, _n in enumerate(("mod", "qkv", "proj", "up", "down")):
+        DOUBLE_IDS[f"{_s}_{_n}_w"] = _i * 10 + 2 * _j
+        DOUBLE_IDS[f"{_s}_{_n}_b"] = _i * 10 + 2 * _j + 1
+WAN_IDS = {"mod_tab": 0, "sa_qkv_w": 1, "sa_qkv_b": 2, "sa_o_w": 3, "sa_o_b": 4,
+           "ca_q_w": 5, "ca_q_b": 6, "ca_kv_w": 7, "ca_kv_b": 8, "ca_o_w": 9, "ca_o_b": 10,
+           "ffn_up_w": 11, "ffn_up_b": 12, "ffn_down_w": 13, "ffn_down_b": 14}
+
+
+def global_shapes(cfg):
+    d, C = cfg["hidden"], cfg["patch_ch"]
+    s = {"pe_w": (d, C), "pe_b": (d,), "t1_w": (d, TEMB_DIM), "t1_b": (d,),
+         "t2_w": (d, d), "t2_b": (d,), "fmod_w": (2 * d, d), "fmod_b": (2 * d,),
+         "fin_w": (C, d), "fin_b": (C,)}
+    if cfg["kind"] == "wan":
+        s["tproj_w"] = (6 * d, d)
+        s["tproj_b"] = (6 * d,)
+    return s
+
+
+def block_shapes(cfg, btype):
+    d, F = cfg["hidden"], cfg["mlp"]
+    if btype == "single":
+        return {"mod_w": (3 * d, d), "mod_b": (3 * d,), "lin1_w": (3 * d + F, d),
+                "lin1_b": (3 * d + F,), "lin2_w": (d, d + F), "lin2_b": (d,)}
+    if btype == "double":
+        s = {}
+        for st in ("img", "txt"):
+            s.update({f"{st}_mod_w": (6 * d, d), f"{st}_mod_b": (6 * d,),
+                      f"{st}_qkv_w": (3 * d, d), f"{st}_qkv_b": (3 * d,),
+                      f"{st}_proj_w": (d, d), f"{st}_proj_b": (d,),
+                      f"{st}_up_w": (F, d), f"{st}_up_b": (F,),
+                      f"{st}_down_w": (d, F), f"{st}_down_b": (d,)})
+        return s
+    if btype == "wan":
+        return {"mod_tab": (6 * d,), "sa_qkv_w": (3 * d, d), "sa_qkv_b": (3 * d,),
+                "sa_o_w": (d, d), "sa_o_b": (d,), "ca_q_w": (d, d), "ca_q_b": (d,),
+                "ca_kv_w": (2 * d, d), "ca_kv_b": (2 * d,), "ca_o_w": (d, d), "ca_o_b": (d,),
+                "ffn_up_w": (F, d), "ffn_up_b": (F,), "ffn_down_w": (d, F),
+                "ffn_down_b": (d,)}
+    raise ValueError(btype)
+
+
+def block_types(cfg):
+    """Block types in execution order."""
+    if cfg["kind"] == "wan":
+        return ["wan"] * cfg["n_wan"]
+    return ["double"] * cfg["n_double"] + ["single"] * cfg["n_single"]
+
+
+def _ids(btype):
+    return {"single": SINGLE_IDS, "double": DOUBLE_IDS, "wan": WAN_IDS}[btype]
+
+
+def _gen(cfg, slot, tid, name, shape):
+    n = int(np.prod(shape))
+    std = BIAS_STD if (name.endswith("_b") or name == "mod_tab") else WEIGHT_STD
+    v = normal(cfg["weight_seed"], slot * 256 + tid, n, std).reshape(shape)
+    # matrices are stored in the GEMM operand type; biases/tables stay fp32
+    if cfg["dtype"] == "bf16" and len(shape) == 2:
+        v = bf16_round(v)
+    return v
+
+
+def make_weights(cfg, blocks=None):
+    """All weights as fp32 numpy arrays (bf16-valued for bf16 configs).
+
+    blocks: optional list of block indices to generate (others are None), so that a
+    reduced-depth oracle run can fetch exactly the blocks it needs."""
+    out = {"global": {}, "blocks": []}
+    for name, shape in global_shapes(cfg).items():
+        out["global"][name] = _gen(cfg, 0, GLOBAL_IDS[name], name, shape)
+    for i, bt in enumerate(block_types(cfg)):
+        if blocks is not None and i not in blocks:
+            out["blocks"].append(None)
+            continue
+        ids = _ids(bt)
+        out["blocks"].append({"type": bt, **{n: _gen(cfg, 1 + i, ids[n], n, s)
+                                             for n, s in block_shapes(cfg, bt).items()}})
+    return out
+
+
+# Gate parameters: MLP 3 -> 16 -> 1 with Xavier-uniform bounds, drawn on the host.
+GATE_IN, GATE_HID = 3, 16
+GATE_KEYS = {"w1": 1, "b1": 2, "w2": 3, "b2": 4}
+
+
+def make_gate(gate_seed):
+    """Seeded gate parameters (fp32): w1 [16,3], b1 [16], w2 [16], b2 [1], mu [3], sd [3]."""
+    a1 = float(np.sqrt(6.0 / (GATE_IN + GATE_HID)))
+    a2 = float(np.sqrt(6.0 / (GATE_HID + 1)))
+    g = {
+        "w1": uniform(gate_seed, GATE_KEYS["w1"], GATE_HID * GATE_IN, -a1, a1).reshape(GATE_HID, GATE_IN),
+        "b1": uniform(gate_seed, GATE_KEYS["b1"], GATE_HID, -0.1, 0.1),
+        "w2": uniform(gate_seed, GATE_KEYS["w2"], GATE_HID, -a2, a2),
+        "b2": uniform(gate_seed, GATE_KEYS["b2"], 1, -0.1, 0.1),
+        "mu": np.zeros(GATE_IN, np.float32),
+        "sd": np.ones(GATE_IN, np.float32),
+    }
+    return g
+
+
+def gate_flat(g):
+    """Flat parameter vector in the order w1 (row-major), b1, w2, b2 (81 floats)."""
+    return np.concatenate([g["w1"].ravel(), g["b1"], g["w2"], g["b2"]]).astype(np.float32)
+
+
+# Sample inputs: latent noise, text tokens and pooled vector, all N(0, 1).
+INPUT_KEYS = {"x": 1, "txt": 2, "pooled": 3}
+
+
+def make_inputs(cfg, sample_seed=0):
+    seed = 1000 + cfg["weight_seed"] * 100 + sample_seed
+    ni, nx, C, d = cfg["n_img"], cfg["n_txt"], cfg["patch_ch"], cfg["hidden"]
+    x = normal(seed, INPUT_KEYS["x"], ni * C, 1.0).reshape(ni, C)
+    txt = normal(seed, INPUT_KEYS["txt"], nx * d, 1.0).reshape(nx, d)
+    pooled = normal(seed, INPUT_KEYS["pooled"], d, 1.0)
+    if cfg["dtype"] == "bf16":
+        txt = bf16_round(txt)
+    return {"x": x, "txt": txt, "pooled": pooled}
