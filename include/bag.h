@@ -1,0 +1,196 @@
+/*
+ * bag.h - C ABI of the GB300 (sm_103a) implementation of BAG's cached DiT sampling path.
+ *
+ * BAG ("Budget-Aware Gating for Diffusion Caching") runs a T-step sampler in which
+ * exactly B steps evaluate the full network and the other T - B reuse the cached
+ * stack residual; a small gate decides each step from the remaining budget and the
+ * trajectory (Sec. 3.1 problem setup, Eq. 1 gate, Eq. 3 state, Algorithm 2).
+ *
+ * Conventions (every entry point):
+ *   - Returns bag_status; nothing throws across the boundary.  On failure the message
+ *     is available from bag_last_error(ctx).  A device-side error (a bounded wait that
+ *     timed out inside a kernel) is sticky: every later call on the context returns
+ *     BAG_EDEVICE_TIMEOUT until bag_reset.
+ *   - "device" pointers are CUDA global-memory pointers on the context's device; "host"
+ *     pointers are ordinary CPU memory.  The library never frees caller memory and never
+ *     keeps a caller pointer past the call that received it.
+ *   - Work is enqueued on the context's stream (bag_set_stream); calls that return
+ *     results in host memory synchronise that stream.  A context is not thread-safe.
+ *   - Tensors are dense row-major.  Image tokens are ordered row-major over the
+ *     (frames, rows, cols) grid; text tokens come first in the joint sequence.
+ */
+#ifndef BAG_H_
+#define BAG_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  BAG_OK = 0,
+  BAG_EINVAL = 1,          /* bad argument (null pointer, size out of range, B > T ...) */
+  BAG_ENOMEM = 2,          /* device allocation failed */
+  BAG_ECUDA = 3,           /* a CUDA runtime call failed (message in bag_last_error) */
+  BAG_EORDER = 4,          /* bag_step called with t != the context's next step */
+  BAG_EDEVICE_TIMEOUT = 5, /* a kernel's bounded wait expired; results are invalid */
+  BAG_ESTATE = 6,          /* call not valid in the context's current state */
+  BAG_EUNSUPPORTED = 7     /* shape/type combination the kernels do not implement */
+} bag_status;
+
+enum { BAG_KIND_SINGLE = 0, BAG_KIND_MMDIT = 1, BAG_KIND_WAN = 2 };
+enum { BAG_F32 = 0, BAG_BF16 = 1 };
+enum {
+  BAG_POLICY_BAG = 0,   /* Algorithm 2: gate decision + the two forced pacing rules */
+  BAG_POLICY_FULL = 1,  /* uncached sampling: every step evaluates the network */
+  BAG_POLICY_MASK = 2   /* follow a caller-given mask (static schedule) */
+};
+
+/* Backbone shape.  kind SINGLE: n_single single-stream blocks on the joint [text; image]
+ * sequence.  MMDIT: n_double double-stream blocks, then n_single single-stream blocks
+ * (FLUX/Qwen-Image layout).  WAN: n_wan blocks of self-attention (3D RoPE),
+ * cross-attention to n_txt context tokens and FFN.  hidden = heads * head_dim;
+ * rope_axes split head_dim over the (frame, row, col) axes (entries even, sum =
+ * head_dim).  dtype: GEMM/attention operand type (the residual stream, latents, the
+ * cached residual and all modulation vectors are fp32 in both cases). */
+typedef struct {
+  int kind;
+  int hidden, heads, mlp;
+  int n_double, n_single, n_wan;
+  int grid[3];        /* frames, rows, cols of image tokens; n_img = product */
+  int n_txt;          /* text tokens (joint attention) or context tokens (Wan) */
+  int patch_ch;       /* latent channels per image token (64) */
+  int rope_axes[3];
+  int dtype;          /* BAG_F32 or BAG_BF16 */
+  uint64_t weight_seed, gate_seed;
+  float tau;          /* gate cutoff: a step computes when sigmoid(z) > tau (0 < tau < 1) */
+} bag_arch;
+
+/* Conditioning of one sample (device pointers, read during bag_step / bag_run).
+ * txt: [n_txt, hidden] text tokens (fp32 for BAG_F32 contexts, bf16 for BAG_BF16).
+ * pooled: [hidden] fp32 pooled text vector added to the time embedding (ignored for
+ * WAN; may be null there). */
+typedef struct {
+  const void* txt;
+  const float* pooled;
+} bag_cond;
+
+/* Per-sample schedule statistics.  mask / log are optional host arrays supplied by the
+ * caller: mask[T] receives m_t, log[T * BAG_LOG_FLOATS] the per-step record
+ *   [0..2] gate inputs (B-c)/B, (T-t)/T, drift;  [3] gate logit z;  [4] raw gate bit;
+ *   [5] m_t;  [6] c before the step;  [7] t - t_last;  [8..10] B/T, (B-c)/B,
+ *   (B-c)/(T-t);  [11] sum|m_t - m_last|;  [12] sum|m_last|.
+ * nfe receives the realised number of full evaluations. */
+#define BAG_LOG_FLOATS 16
+typedef struct {
+  uint8_t* mask;
+  float* log;
+  int nfe;
+  int T, B;
+} bag_stats;
+
+typedef struct bag_ctx bag_ctx;
+
+/* Create a context for `arch` with a T-step sampler under budget B (1 <= B <= T,
+ * Sec. 3.1: ||m||_1 = B with m_0 = 1).  Allocates and seeds all weights on the current
+ * CUDA device from arch->weight_seed (SplitMix64 counter generator), seeds the gate
+ * from arch->gate_seed, and allocates every activation buffer the step needs, so that
+ * no later call allocates.  *out receives the context (NULL on failure).
+ * Errors: EINVAL (bad arch/T/B), ENOMEM, ECUDA, EUNSUPPORTED. */
+bag_status bag_create(const bag_arch* arch, int T, int B, bag_ctx** out);
+
+/* Release every device resource of the context (null is a no-op). */
+void bag_destroy(bag_ctx* ctx);
+
+/* Text of the last error on this context (or of the last failed bag_create when ctx is
+ * null).  Valid until the next call on the context. */
+const char* bag_last_error(bag_ctx* ctx);
+
+/* Make later work run on `cuda_stream` (a cudaStream_t; null = the legacy stream).
+ * Invalidates captured step graphs (they are re-captured on first use). */
+bag_status bag_set_stream(bag_ctx* ctx, void* cuda_stream);
+
+/* Replace the gate parameters (Eq. 1; App. A.2 z-scored inputs).  theta: host array of
+ * 81 floats = W1[16][3] row-major, b1[16], w2[16], b2; mu, sd: host arrays of 3 floats
+ * (z-score statistics; null = 0 and 1). */
+bag_status bag_load_gate(bag_ctx* ctx, const float* theta, const float* mu, const float* sd);
+
+/* Choose the schedule policy (BAG_POLICY_*).  For BAG_POLICY_MASK, host_mask[T] gives
+ * the per-step bits (host_mask[0] is ignored: step 0 always computes).  The budget
+ * pacing of Algorithm 2 applies only to BAG_POLICY_BAG. */
+bag_status bag_set_policy(bag_ctx* ctx, int policy, const uint8_t* host_mask);
+
+/* Start a new sample: t = 0, c = 0, cache invalid, sticky device error cleared. */
+bag_status bag_reset(bag_ctx* ctx);
+
+/* One sampler step (Algorithm 2, one iteration).  t must equal the context's next step
+ * (0, 1, ..., T-1 after bag_reset) else EORDER.  x: device fp32 [n_img, patch_ch]
+ * latent x_t; x_out: device fp32 [n_img, patch_ch] receives x_{t+1} (may equal x).
+ * full_or_cached: device int32* written asynchronously with 1 (full evaluation) or 0
+ * (cached residual reused); may be null.  The decision is taken on the device: no host
+ * synchronisation happens inside the step. */
+bag_status bag_step(bag_ctx* ctx, const float* x, int t, const bag_cond* cond, float* x_out,
+                    int32_t* full_or_cached);
+
+/* All T steps of one sample from the context's current state (normally right after
+ * bag_reset), in place on x_inout (device fp32 [n_img, patch_ch]).  stats (optional,
+ * host) receives the schedule after one synchronisation at the end. */
+bag_status bag_run(bag_ctx* ctx, float* x_inout, const bag_cond* cond, bag_stats* stats);
+
+/* Same as bag_run with HOST buffers: copies x (fp32 [n_img, patch_ch]), txt (fp32
+ * [n_txt, hidden], converted on device for bf16 contexts) and pooled (fp32 [hidden],
+ * may be null for WAN) to the device, runs the sample and copies the result back into
+ * x_host.  For pageable memory the copies are synchronous. */
+bag_status bag_run_host(bag_ctx* ctx, float* x_host, const float* txt_host,
+                        const float* pooled_host, bag_stats* stats);
+
+/* ---- inspection and single-operation entry points (tests, benchmarks) ---- */
+
+/* Copy weight tensor `name` of block `block` (-1 = global tensors) to host fp32
+ * `out` (n elements, must equal the tensor size).  Names follow the seeded generator's
+ * inventory (e.g. "lin1_w", "img_qkv_b", "pe_w", "fmod_w"). */
+bag_status bag_get_weight(bag_ctx* ctx, int block, const char* name, float* out, size_t n);
+
+/* Run block `block` of the stack once on a caller-provided stream state, with the
+ * modulation of step t_mod of the current sample (modulation is precomputed by
+ * bag_prepare).  h: device fp32 joint sequence [n_txt + n_img, hidden] (text rows first)
+ * for SINGLE/MMDIT; for WAN h is the image stream [n_img, hidden] and the context comes
+ * from the last bag_prepare.  Updated in place. */
+bag_status bag_forward_block(bag_ctx* ctx, int block, int t_mod, float* h);
+
+/* Precompute the conditioning of a sample (time embedding and every block's
+ * modulation for all T steps) and stage its text tokens; bag_run does this itself. */
+bag_status bag_prepare(bag_ctx* ctx, const bag_cond* cond);
+
+/* Number of kernel launches the last bag_run enqueued (graph nodes included). */
+bag_status bag_launch_count(bag_ctx* ctx, long* out);
+
+/* C[M,N] = A[M,K] W[N,K]^T (+ bias[N]) on the tensor cores: A, W bf16 device, lda/ldw
+ * in elements (multiples of 8), K a multiple of 64, N a multiple of 64; C fp32 device
+ * with row stride ldc; bias device fp32 or null.  epilogue: 0 = store, 1 = GELU(tanh).
+ * force_simt != 0 runs the CUDA-core kernel instead (cross-check). */
+bag_status bag_gemm_bf16(bag_ctx* ctx, const void* A, long lda, const void* W, long ldw,
+                         const float* bias, float* C, long ldc, int M, int N, int K,
+                         int epilogue, int force_simt);
+
+/* Multi-head attention softmax(q k^T / sqrt(dh)) v: q [nq, ld], k, v [nk, ld] bf16 device,
+ * head h at columns [h*dh, (h+1)*dh); o [nq, ld] bf16 device.  dh = 64 or 128. */
+bag_status bag_attention_bf16(bag_ctx* ctx, const void* q, const void* k, const void* v,
+                              void* o, long ld, int nq, int nk, int heads, int dh,
+                              int force_simt);
+
+/* y = (1 + scale) * LayerNorm(x) + shift row-wise (eps 1e-6, no affine): x fp32 device
+ * [rows, cols], shift/scale fp32 device [cols] (null = plain LayerNorm), y bf16 device. */
+bag_status bag_ln_mod(bag_ctx* ctx, const float* x, const float* shift, const float* scale,
+                      void* y, int rows, int cols);
+
+/* Skip path (plain residual reuse): out = h_in + R, fp32 device, n elements (n % 4 == 0). */
+bag_status bag_residual_add(bag_ctx* ctx, float* out, const float* h_in, const float* R, long n);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BAG_H_ */

@@ -1,0 +1,1388 @@
+// C ABI of the BAG sampler: context (weights, activation arena, device state), the
+// per-sample conditioning precompute, one denoising step as a CUDA graph whose
+// full-network body and residual-reuse body hang off a conditional node that the gate
+// kernel sets on the device, and the single-operation entry points.
+//
+// One step, as enqueued (Algorithm 2, one iteration):
+//   prefix : patch embed  h_in = x W_pe^T + b  (also seeds the image stream)
+//            signal       m_t = LN-mod of h_in with block 0's first modulation, fused with
+//                         the per-row partial sums of |m_t - m_last| and |m_last|
+//            gate         drift, gate MLP, forced rules, counters, log, decision
+//   full   : text tokens -> stream, every block, R = h_out - h_in, m_last <- m_t
+//   reuse  : h_out = h_in + R
+//   suffix : final LN-mod + projection fused with the Euler update, t += 1
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <string>
+#include <vector>
+
+#include "bag.h"
+#include "kernels.h"
+
+using namespace bag;
+
+namespace {
+
+struct Tensor {
+  void* p = nullptr;
+  long n = 0;
+  int bf16 = 0;
+};
+
+enum BlockType { BT_SINGLE = 0, BT_DOUBLE = 1, BT_WAN = 2 };
+
+struct Block {
+  int type = BT_SINGLE;
+  std::map<std::string, Tensor> w;
+  long mod_off = 0;  // column of this block's first modulation vector in a mod_all row
+};
+
+// ----- the seeded generator, host side (SplitMix64; same definition as the device fill)
+uint64_t sm_mix(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+uint64_t sm_start(uint64_t seed, uint64_t key) {
+  return sm_mix((seed * 0x9E3779B97F4A7C15ull) ^ sm_mix(key));
+}
+void sm_uniform(uint64_t seed, uint64_t key, int n, double lo, double hi, float* out) {
+  const uint64_t s = sm_start(seed, key);
+  const float lo32 = (float)lo, hi32 = (float)hi;
+  const float span = hi32 - lo32;
+  for (int i = 0; i < n; ++i) {
+    const uint64_t u = sm_mix(s + (uint64_t)(i + 1) * 0x9E3779B97F4A7C15ull);
+    const float f = (float)(u >> 40) * (1.0f / 16777216.0f);
+    const float prod = span * f;
+    out[i] = lo32 + prod;
+  }
+}
+
+// Tensor ids of the generator's inventory (key = slot * 256 + id).
+const std::map<std::string, int> kGlobalIds = {
+    {"pe_w", 0}, {"pe_b", 1}, {"t1_w", 2}, {"t1_b", 3}, {"t2_w", 4}, {"t2_b", 5},
+    {"fmod_w", 6}, {"fmod_b", 7}, {"fin_w", 8}, {"fin_b", 9}, {"tproj_w", 10}, {"tproj_b", 11}};
+const std::map<std::string, int> kSingleIds = {{"mod_w", 0}, {"mod_b", 1}, {"lin1_w", 2},
+                                               {"lin1_b", 3}, {"lin2_w", 4}, {"lin2_b", 5}};
+std::map<std::string, int> double_ids() {
+  std::map<std::string, int> m;
+  const char* st[2] = {"img", "txt"};
+  const char* nm[5] = {"mod", "qkv", "proj", "up", "down"};
+  for (int i = 0; i < 2; ++i)
+    for (int j = 0; j < 5; ++j) {
+      m[std::string(st[i]) + "_" + nm[j] + "_w"] = i * 10 + 2 * j;
+      m[std::string(st[i]) + "_" + nm[j] + "_b"] = i * 10 + 2 * j + 1;
+    }
+  return m;
+}
+const std::map<std::string, int> kWanIds = {
+    {"mod_tab", 0}, {"sa_qkv_w", 1}, {"sa_qkv_b", 2}, {"sa_o_w", 3}, {"sa_o_b", 4},
+    {"ca_q_w", 5}, {"ca_q_b", 6}, {"ca_kv_w", 7}, {"ca_kv_b", 8}, {"ca_o_w", 9}, {"ca_o_b", 10},
+    {"ffn_up_w", 11}, {"ffn_up_b", 12}, {"ffn_down_w", 13}, {"ffn_down_b", 14}};
+
+constexpr int kTembDim = 256;
+constexpr int kGateFloats = 87;
+
+}  // namespace
+
+struct bag_ctx {
+  bag_arch arch{};
+  int T = 0, B = 0;
+  int d = 0, H = 0, dh = 0, F = 0, C = 0, ni = 0, nx = 0, N = 0, nrope = 0, nblk = 0;
+  int act_bf16 = 0;
+  size_t act_size = 4;
+  cudaStream_t stream = nullptr;       // internal stream: all work and graph capture
+  cudaStream_t user_stream = nullptr;  // caller's stream (bag_set_stream), bridged by events
+  cudaEvent_t ev_in = nullptr, ev_out = nullptr;
+  std::string err;
+
+  // weights
+  void* warena = nullptr;
+  std::map<std::string, Tensor> G;
+  std::vector<Block> blocks;
+  Tensor wmod;        // [n_mod, d]: every modulation projection, concatenated
+  float* bmod = nullptr;
+  long n_mod = 0;
+  long mod_stride = 0;  // floats per step in mod_all
+  long fmod_off = 0;    // final-layer modulation column in mod_all
+  float* wan_tabs = nullptr;  // [nblk][6d]
+
+  // gate
+  float* d_gate = nullptr;
+  float thr = 0.f;
+  int policy = BAG_POLICY_BAG;
+  uint8_t* d_pmask = nullptr;
+
+  // activations
+  void* aarena = nullptr;
+  float *x = nullptr, *h_in = nullptr, *hj = nullptr, *R = nullptr;
+  void *m_cur = nullptr, *m_last = nullptr;
+  float* sig_partial = nullptr;
+  __nv_bfloat16* xb = nullptr;
+  void *xn = nullptr, *q = nullptr, *k = nullptr, *vt = nullptr, *cat = nullptr;
+  void *qc = nullptr, *kc = nullptr, *vtc = nullptr;
+  long vpad = 0, vpad_c = 0;
+  void* txt_stage = nullptr;
+  float* pooled_stage = nullptr;
+  float2* rope = nullptr;
+  float* dsig = nullptr;
+  void *sin_all = nullptr, *t1o = nullptr, *svec = nullptr;
+  float *vec_all = nullptr, *mod_all = nullptr, *wan_shared = nullptr;
+  DevState* st = nullptr;     // sampler state
+  DevState* st_op = nullptr;  // state for single-operation calls
+  float* log = nullptr;
+  float* tmp_f32 = nullptr;   // staging for bag_run_host text conversion
+  long tmp_f32_n = 0;
+
+  // step graph
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t exec = nullptr;
+  cudaStream_t cap_stream = nullptr;
+  int use_graph = 1;
+  long n_prefix = 0, n_full = 0, n_skip = 0, n_suffix = 0, n_prepare = 0;
+  long launches = 0;
+
+  int next_t = 0;
+  bool prepared = false;
+};
+
+static std::string g_create_error;
+
+#define CK(expr)                                                                     \
+  do {                                                                               \
+    cudaError_t _e = (expr);                                                         \
+    if (_e != cudaSuccess) {                                                         \
+      ctx->err = std::string(#expr) + ": " + cudaGetErrorString(_e);                 \
+      return BAG_ECUDA;                                                              \
+    }                                                                                \
+  } while (0)
+
+#define CKS(expr)                                  \
+  do {                                             \
+    bag_status _s = (expr);                        \
+    if (_s != BAG_OK) return _s;                   \
+  } while (0)
+
+static bag_status fail(bag_ctx* ctx, bag_status s, const std::string& msg) {
+  if (ctx)
+    ctx->err = msg;
+  else
+    g_create_error = msg;
+  return s;
+}
+
+// ---------------------------------------------------------------------------
+// creation
+// ---------------------------------------------------------------------------
+static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+namespace {
+struct Arena {
+  size_t off = 0;
+  std::vector<std::pair<void**, size_t>> items;
+  void add(void** slot, size_t bytes) {
+    items.push_back({slot, off});
+    off += align256(bytes);
+  }
+  void bind(char* base) {
+    for (auto& it : items) *it.first = base + it.second;
+  }
+};
+}  // namespace
+
+static bag_status validate_arch(const bag_arch* a, int T, int B) {
+  if (!a) return fail(nullptr, BAG_EINVAL, "arch is null");
+  if (T < 1 || B < 1 || B > T) return fail(nullptr, BAG_EINVAL, "need 1 <= B <= T");
+  if (a->kind < 0 || a->kind > 2) return fail(nullptr, BAG_EINVAL, "unknown kind");
+  if (a->hidden <= 0 || a->heads <= 0 || a->hidden % a->heads) return fail(nullptr, BAG_EINVAL, "hidden % heads");
+  const int dh = a->hidden / a->heads;
+  if (dh != 64 && dh != 128) return fail(nullptr, BAG_EUNSUPPORTED, "head_dim must be 64 or 128");
+  if (a->hidden % 64 || a->mlp % 64 || a->mlp <= 0) return fail(nullptr, BAG_EUNSUPPORTED, "hidden and mlp must be multiples of 64");
+  if (a->hidden > 6144) return fail(nullptr, BAG_EUNSUPPORTED, "hidden > 6144");
+  if (a->patch_ch != 64) return fail(nullptr, BAG_EUNSUPPORTED, "patch_ch must be 64");
+  if (a->grid[0] < 1 || a->grid[1] < 1 || a->grid[2] < 1 || a->n_txt < 1) return fail(nullptr, BAG_EINVAL, "empty grid or text");
+  int s = 0;
+  for (int i = 0; i < 3; ++i) {
+    if (a->rope_axes[i] < 0 || a->rope_axes[i] % 2) return fail(nullptr, BAG_EINVAL, "rope axes must be even");
+    s += a->rope_axes[i];
+  }
+  if (s != dh) return fail(nullptr, BAG_EINVAL, "rope axes must sum to head_dim");
+  const int nb = a->kind == BAG_KIND_WAN ? a->n_wan : a->n_double + a->n_single;
+  if (nb < 1) return fail(nullptr, BAG_EINVAL, "no blocks");
+  if (a->kind == BAG_KIND_SINGLE && a->n_double) return fail(nullptr, BAG_EINVAL, "SINGLE kind has no double blocks");
+  if (!(a->tau > 0.f && a->tau < 1.f)) return fail(nullptr, BAG_EINVAL, "tau must be in (0, 1)");
+  if (a->dtype != BAG_F32 && a->dtype != BAG_BF16) return fail(nullptr, BAG_EINVAL, "dtype");
+  return BAG_OK;
+}
+
+static std::map<std::string, std::vector<long>> global_shapes(const bag_ctx* c) {
+  const long d = c->d, C = c->C;
+  std::map<std::string, std::vector<long>> s = {
+      {"pe_w", {d, C}}, {"pe_b", {d}}, {"t1_w", {d, kTembDim}}, {"t1_b", {d}}, {"t2_w", {d, d}},
+      {"t2_b", {d}}, {"fmod_w", {2 * d, d}}, {"fmod_b", {2 * d}}, {"fin_w", {C, d}}, {"fin_b", {C}}};
+  if (c->arch.kind == BAG_KIND_WAN) {
+    s["tproj_w"] = {6 * d, d};
+    s["tproj_b"] = {6 * d};
+  }
+  return s;
+}
+
+static std::map<std::string, std::vector<long>> block_shapes(const bag_ctx* c, int type) {
+  const long d = c->d, F = c->F;
+  if (type == BT_SINGLE)
+    return {{"mod_w", {3 * d, d}}, {"mod_b", {3 * d}}, {"lin1_w", {3 * d + F, d}},
+            {"lin1_b", {3 * d + F}}, {"lin2_w", {d, d + F}}, {"lin2_b", {d}}};
+  if (type == BT_DOUBLE) {
+    std::map<std::string, std::vector<long>> s;
+    for (const char* st : {"img", "txt"}) {
+      std::string p(st);
+      s[p + "_mod_w"] = {6 * d, d};
+      s[p + "_mod_b"] = {6 * d};
+      s[p + "_qkv_w"] = {3 * d, d};
+      s[p + "_qkv_b"] = {3 * d};
+      s[p + "_proj_w"] = {d, d};
+      s[p + "_proj_b"] = {d};
+      s[p + "_up_w"] = {F, d};
+      s[p + "_up_b"] = {F};
+      s[p + "_down_w"] = {d, F};
+      s[p + "_down_b"] = {d};
+    }
+    return s;
+  }
+  return {{"mod_tab", {6 * d}}, {"sa_qkv_w", {3 * d, d}}, {"sa_qkv_b", {3 * d}},
+          {"sa_o_w", {d, d}}, {"sa_o_b", {d}}, {"ca_q_w", {d, d}}, {"ca_q_b", {d}},
+          {"ca_kv_w", {2 * d, d}}, {"ca_kv_b", {2 * d}}, {"ca_o_w", {d, d}}, {"ca_o_b", {d}},
+          {"ffn_up_w", {F, d}}, {"ffn_up_b", {F}}, {"ffn_down_w", {d, F}}, {"ffn_down_b", {d}}};
+}
+
+static bool is_mod_weight(const std::string& n) {
+  return n == "mod_w" || n == "img_mod_w" || n == "txt_mod_w";
+}
+static bool is_mod_bias(const std::string& n) {
+  return n == "mod_b" || n == "img_mod_b" || n == "txt_mod_b";
+}
+
+static bag_status alloc_weights(bag_ctx* ctx) {
+  const int act = ctx->act_bf16;
+  const long d = ctx->d;
+  // modulation projections first, contiguous: [blocks..., final] (Wan: [tproj, final])
+  std::vector<std::pair<std::string, int>> mod_order;  // (name, block or -1)
+  long nmod = 0;
+  for (int b = 0; b < ctx->nblk; ++b) {
+    Block& blk = ctx->blocks[b];
+    if (blk.type == BT_DOUBLE) {
+      blk.mod_off = nmod;
+      mod_order.push_back({"img_mod", b});
+      mod_order.push_back({"txt_mod", b});
+      nmod += 12 * d;
+    } else if (blk.type == BT_SINGLE) {
+      blk.mod_off = nmod;
+      mod_order.push_back({"mod", b});
+      nmod += 3 * d;
+    } else {
+      blk.mod_off = (long)b * 6 * d;
+    }
+  }
+  if (ctx->arch.kind == BAG_KIND_WAN) {
+    mod_order.push_back({"tproj", -1});
+    ctx->fmod_off = (long)ctx->nblk * 6 * d;
+    ctx->mod_stride = ctx->fmod_off + 2 * d;
+    nmod = 6 * d;
+  } else {
+    ctx->fmod_off = nmod;
+    ctx->mod_stride = nmod + 2 * d;
+  }
+  mod_order.push_back({"fmod", -1});
+  nmod += 2 * d;
+  ctx->n_mod = nmod;
+
+  // sizes
+  size_t total = 0;
+  const size_t es = act ? 2 : 4;
+  total += align256((size_t)nmod * d * es) + align256((size_t)nmod * 4);
+  auto gs = global_shapes(ctx);
+  for (auto& kv : gs) {
+    if (kv.first == "fmod_w" || kv.first == "fmod_b" || kv.first == "tproj_w" || kv.first == "tproj_b") continue;
+    long n = 1;
+    for (long v : kv.second) n *= v;
+    total += align256((size_t)n * (kv.second.size() == 2 ? es : 4));
+  }
+  for (int b = 0; b < ctx->nblk; ++b) {
+    for (auto& kv : block_shapes(ctx, ctx->blocks[b].type)) {
+      if (is_mod_weight(kv.first) || is_mod_bias(kv.first)) continue;
+      long n = 1;
+      for (long v : kv.second) n *= v;
+      total += align256((size_t)n * (kv.second.size() == 2 ? es : 4));
+    }
+  }
+  if (cudaMalloc(&ctx->warena, total) != cudaSuccess)
+    return fail(ctx, BAG_ENOMEM, "weight allocation of " + std::to_string(total) + " bytes failed");
+  char* base = (char*)ctx->warena;
+  size_t off = 0;
+  ctx->wmod = {base, nmod * d, act};
+  off += align256((size_t)nmod * d * es);
+  ctx->bmod = (float*)(base + off);
+  off += align256((size_t)nmod * 4);
+  // bind modulation pieces into the concatenated buffers
+  long row = 0;
+  for (auto& it : mod_order) {
+    const std::string& stem = it.first;
+    const long rows = stem == "fmod" ? 2 * d : (stem == "mod" ? 3 * d : 6 * d);
+    Tensor w{(char*)ctx->wmod.p + (size_t)row * d * es, rows * d, act};
+    Tensor bb{ctx->bmod + row, rows, 0};
+    if (it.second < 0) {
+      ctx->G[stem + "_w"] = w;
+      ctx->G[stem + "_b"] = bb;
+    } else {
+      ctx->blocks[it.second].w[stem + "_w"] = w;
+      ctx->blocks[it.second].w[stem + "_b"] = bb;
+    }
+    row += rows;
+  }
+  for (auto& kv : gs) {
+    if (ctx->G.count(kv.first)) continue;
+    long n = 1;
+    for (long v : kv.second) n *= v;
+    const int is_mat = kv.second.size() == 2;
+    ctx->G[kv.first] = {base + off, n, is_mat ? act : 0};
+    off += align256((size_t)n * (is_mat ? es : 4));
+  }
+  // Wan per-block tables go contiguous for the expansion kernel
+  if (ctx->arch.kind == BAG_KIND_WAN) {
+    ctx->wan_tabs = (float*)(base + off);
+    for (int b = 0; b < ctx->nblk; ++b) ctx->blocks[b].w["mod_tab"] = {ctx->wan_tabs + (size_t)b * 6 * d, 6 * d, 0};
+    off += align256((size_t)ctx->nblk * 6 * d * 4);
+  }
+  for (int b = 0; b < ctx->nblk; ++b) {
+    for (auto& kv : block_shapes(ctx, ctx->blocks[b].type)) {
+      if (ctx->blocks[b].w.count(kv.first)) continue;
+      long n = 1;
+      for (long v : kv.second) n *= v;
+      const int is_mat = kv.second.size() == 2;
+      ctx->blocks[b].w[kv.first] = {base + off, n, is_mat ? act : 0};
+      off += align256((size_t)n * (is_mat ? es : 4));
+    }
+  }
+  if (off > total) return fail(ctx, BAG_ESTATE, "weight arena overflow");
+  return BAG_OK;
+}
+
+static bag_status seed_weights(bag_ctx* ctx) {
+  const uint64_t seed = ctx->arch.weight_seed;
+  auto fill = [&](const Tensor& t, int slot, int id, bool is_bias) -> bag_status {
+    const double sd = 0.02;  // weights and biases N(0, 0.02) (Irwin-Hall(4) approximation)
+    const float c32 = (float)(sd * std::sqrt(3.0) / 65536.0);
+    (void)is_bias;
+    cudaError_t e = fill_synth(t.p, t.n, sm_start(seed, (uint64_t)slot * 256 + id), 0, c32, t.bf16,
+                               ctx->stream);
+    if (e != cudaSuccess) return fail(ctx, BAG_ECUDA, std::string("fill: ") + cudaGetErrorString(e));
+    return BAG_OK;
+  };
+  for (auto& kv : ctx->G) {
+    auto it = kGlobalIds.find(kv.first);
+    if (it == kGlobalIds.end()) return fail(ctx, BAG_ESTATE, "unknown global " + kv.first);
+    CKS(fill(kv.second, 0, it->second, false));
+  }
+  const auto dids = double_ids();
+  for (int b = 0; b < ctx->nblk; ++b) {
+    const Block& blk = ctx->blocks[b];
+    const std::map<std::string, int>& ids =
+        blk.type == BT_SINGLE ? kSingleIds : (blk.type == BT_DOUBLE ? dids : kWanIds);
+    for (auto& kv : blk.w) {
+      auto it = ids.find(kv.first);
+      if (it == ids.end()) return fail(ctx, BAG_ESTATE, "unknown block tensor " + kv.first);
+      CKS(fill(kv.second, 1 + b, it->second, false));
+    }
+  }
+  return BAG_OK;
+}
+
+static bag_status seed_gate(bag_ctx* ctx) {
+  float g[kGateFloats];
+  const uint64_t s = ctx->arch.gate_seed;
+  const double a1 = std::sqrt(6.0 / 19.0), a2 = std::sqrt(6.0 / 17.0);
+  sm_uniform(s, 1, 48, -a1, a1, g);
+  sm_uniform(s, 2, 16, -0.1, 0.1, g + 48);
+  sm_uniform(s, 3, 16, -a2, a2, g + 64);
+  sm_uniform(s, 4, 1, -0.1, 0.1, g + 80);
+  for (int i = 0; i < 3; ++i) {
+    g[81 + i] = 0.f;
+    g[84 + i] = 1.f;
+  }
+  CK(cudaMemcpy(ctx->d_gate, g, sizeof(g), cudaMemcpyHostToDevice));
+  return BAG_OK;
+}
+
+static void rope_table(const bag_ctx* ctx, std::vector<float2>& tab) {
+  // angle of pair j (axes laid out one after another) at token position p:
+  // p_axis * theta^(-2 jj / d_axis)
+  const int half = ctx->dh / 2;
+  tab.assign((size_t)ctx->nrope * half, make_float2(1.f, 0.f));
+  const int f = ctx->arch.grid[0], r = ctx->arch.grid[1], c = ctx->arch.grid[2];
+  const int txt_rows = ctx->arch.kind == BAG_KIND_WAN ? 0 : ctx->nx;
+  for (int row = 0; row < ctx->nrope; ++row) {
+    double pos[3] = {0, 0, 0};
+    if (row >= txt_rows) {
+      const int i = row - txt_rows;
+      pos[0] = i / (r * c);
+      pos[1] = (i / c) % r;
+      pos[2] = i % c;
+    }
+    int j = 0;
+    for (int a = 0; a < 3; ++a) {
+      const int da = ctx->arch.rope_axes[a];
+      for (int jj = 0; jj < da / 2; ++jj, ++j) {
+        const double ang = pos[a] * std::pow(10000.0, -2.0 * jj / da);
+        tab[(size_t)row * half + j] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+      }
+    }
+  }
+  (void)f;
+}
+
+static bag_status alloc_activations(bag_ctx* ctx) {
+  const size_t es = ctx->act_size;
+  const long d = ctx->d, F = ctx->F, ni = ctx->ni, nx = ctx->nx, N = ctx->N, T = ctx->T;
+  const bool wan = ctx->arch.kind == BAG_KIND_WAN;
+  ctx->vpad = ((long)ctx->nrope + 127) / 128 * 128;
+  ctx->vpad_c = ((long)nx + 127) / 128 * 128;
+  const long rows = wan ? ni : N;
+  Arena A;
+  A.add((void**)&ctx->x, (size_t)ni * ctx->C * 4);
+  A.add((void**)&ctx->xb, (size_t)ni * ctx->C * 2);
+  A.add((void**)&ctx->h_in, (size_t)ni * d * 4);
+  A.add((void**)&ctx->hj, (size_t)rows * d * 4);
+  A.add((void**)&ctx->R, (size_t)ni * d * 4);
+  A.add(&ctx->m_cur, (size_t)ni * d * es);
+  A.add(&ctx->m_last, (size_t)ni * d * es);
+  A.add((void**)&ctx->sig_partial, (size_t)ni * 2 * 4);
+  A.add(&ctx->xn, (size_t)rows * d * es);
+  A.add(&ctx->q, (size_t)rows * d * es);
+  A.add(&ctx->k, (size_t)rows * d * es);
+  A.add(&ctx->vt, std::max((size_t)rows * d, (size_t)d * ctx->vpad) * es);
+  A.add(&ctx->cat, (size_t)rows * (d + F) * es);
+  if (wan) {
+    A.add(&ctx->qc, (size_t)ni * d * es);
+    A.add(&ctx->kc, (size_t)nx * d * es);
+    A.add(&ctx->vtc, std::max((size_t)nx * d, (size_t)d * ctx->vpad_c) * es);
+  }
+  A.add(&ctx->txt_stage, (size_t)nx * d * es);
+  A.add((void**)&ctx->pooled_stage, (size_t)d * 4);
+  A.add((void**)&ctx->rope, (size_t)ctx->nrope * (ctx->dh / 2) * sizeof(float2));
+  A.add((void**)&ctx->dsig, (size_t)T * 4);
+  A.add(&ctx->sin_all, (size_t)T * kTembDim * es);
+  A.add(&ctx->t1o, (size_t)T * d * es);
+  A.add(&ctx->svec, (size_t)T * d * es);
+  A.add((void**)&ctx->vec_all, (size_t)T * d * 4);
+  A.add((void**)&ctx->mod_all, (size_t)T * ctx->mod_stride * 4);
+  if (wan) A.add((void**)&ctx->wan_shared, (size_t)T * 8 * d * 4);
+  A.add((void**)&ctx->st, sizeof(DevState));
+  A.add((void**)&ctx->st_op, sizeof(DevState));
+  A.add((void**)&ctx->log, (size_t)T * kLogFloats * 4);
+  A.add((void**)&ctx->d_gate, kGateFloats * 4);
+  A.add((void**)&ctx->d_pmask, (size_t)T);
+  ctx->tmp_f32_n = (long)nx * d;
+  A.add((void**)&ctx->tmp_f32, (size_t)ctx->tmp_f32_n * 4);
+  if (cudaMalloc(&ctx->aarena, A.off) != cudaSuccess)
+    return fail(ctx, BAG_ENOMEM, "activation allocation of " + std::to_string(A.off) + " bytes failed");
+  A.bind((char*)ctx->aarena);
+  CK(cudaMemset(ctx->aarena, 0, A.off));
+  std::vector<float2> tab;
+  rope_table(ctx, tab);
+  CK(cudaMemcpy(ctx->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice));
+  std::vector<float> ds(T);
+  for (int t = 0; t < T; ++t) {
+    const double s0 = 1.0 - (double)t / T, s1 = 1.0 - (double)(t + 1) / T;
+    ds[t] = (float)(s1 - s0);
+  }
+  CK(cudaMemcpy(ctx->dsig, ds.data(), T * 4, cudaMemcpyHostToDevice));
+  return BAG_OK;
+}
+
+// ---------------------------------------------------------------------------
+// enqueue helpers
+// ---------------------------------------------------------------------------
+struct Enq {
+  bag_ctx* ctx;
+  cudaStream_t s;
+  long* count;
+  cudaError_t e = cudaSuccess;
+  void chk(cudaError_t r) {
+    if (e == cudaSuccess && r != cudaSuccess) e = r;
+    if (count) ++*count;
+  }
+};
+
+static Epi base_epi(const bag_ctx* ctx, const DevState* st, int flag_want) {
+  Epi e;
+  e.st = st;
+  e.flag_want = flag_want;
+  e.act_bf16 = ctx->act_bf16;
+  return e;
+}
+
+static inline void* off_act(const bag_ctx* ctx, void* p, long elems) {
+  return (char*)p + elems * (long)ctx->act_size;
+}
+
+static void enq_gemm(Enq& q, const void* A, long lda, const Tensor& W, long ldw, int M, int N,
+                     int K, const Epi& e) {
+  q.chk(gemm(A, lda, W.p, ldw, M, N, K, q.ctx->act_bf16, e, q.ctx->st ? &q.ctx->st->err : nullptr, q.s));
+}
+
+static void enq_ln(Enq& q, const float* x, long ldx, void* y, long ldy, int rows, int split,
+                   const float* sh_a, const float* sc_a, const float* sh_b, const float* sc_b,
+                   const DevState* st, int flag_want) {
+  LnArgs a{};
+  a.x = x;
+  a.ldx = ldx;
+  a.y = y;
+  a.ldy = ldy;
+  a.y_bf16 = q.ctx->act_bf16;
+  a.rows = rows;
+  a.cols = q.ctx->d;
+  a.split = split;
+  a.shift_a = sh_a;
+  a.scale_a = sc_a;
+  a.shift_b = sh_b;
+  a.scale_b = sc_b;
+  a.mod_step = q.ctx->mod_stride;
+  a.st = st;
+  a.flag_want = flag_want;
+  q.chk(ln_mod(a, q.s));
+}
+
+static void enq_qkv_epi(const bag_ctx* ctx, Epi& e, int row_off, bool rope) {
+  e.kind = EPI_QKV;
+  e.q = ctx->q;
+  e.k = ctx->k;
+  e.v = ctx->vt;
+  e.v_mode = ctx->act_bf16 ? 1 : 0;
+  e.vpad = ctx->vpad;
+  e.ldqk = ctx->d;
+  e.d = ctx->d;
+  e.dh = ctx->dh;
+  e.row_off = row_off;
+  e.col_base = 0;
+  e.rope = rope ? ctx->rope : nullptr;
+  e.mlp = off_act(ctx, ctx->cat, ctx->d);
+  e.ldm = ctx->d + ctx->F;
+}
+
+static void enq_attn(Enq& q, const void* Q, const void* K, const void* V, long vpad, void* O,
+                     long ldo, int nq, int nk, const DevState* st, int flag_want) {
+  const bag_ctx* ctx = q.ctx;
+  AttnArgs a{};
+  a.q = Q;
+  a.ldq = ctx->d;
+  a.k = K;
+  a.ldk = ctx->d;
+  a.v = V;
+  a.v_mode = ctx->act_bf16 ? 1 : 0;
+  a.ldv = ctx->d;
+  a.vpad = vpad;
+  a.o = O;
+  a.ldo = ldo;
+  a.nq = nq;
+  a.nk = nk;
+  a.heads = ctx->H;
+  a.dh = ctx->dh;
+  a.bf16 = ctx->act_bf16;
+  a.st = st;
+  a.flag_want = flag_want;
+  q.chk(attention(a, ctx->st ? &ctx->st->err : nullptr, q.s));
+}
+
+// One block of the stack on the stream h (joint [N, d] with text rows first, or the
+// Wan image stream [ni, d]).
+static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw) {
+  bag_ctx* ctx = q.ctx;
+  const Block& blk = ctx->blocks[b];
+  const long d = ctx->d, F = ctx->F, ldc = d + F;
+  const int ni = ctx->ni, nx = ctx->nx, N = ctx->N;
+  const float* mod = ctx->mod_all + blk.mod_off;
+  const long ms = ctx->mod_stride;
+  if (blk.type == BT_SINGLE) {
+    enq_ln(q, h, d, ctx->xn, d, N, 0, mod, mod + d, mod, mod + d, st, fw);
+    Epi e = base_epi(ctx, st, fw);
+    enq_qkv_epi(ctx, e, 0, true);
+    enq_gemm(q, ctx->xn, d, blk.w.at("lin1_w"), d, N, (int)(3 * d + F), (int)d,
+             (e.bias = (const float*)blk.w.at("lin1_b").p, e));
+    enq_attn(q, ctx->q, ctx->k, ctx->vt, ctx->vpad, ctx->cat, ldc, N, N, st, fw);
+    Epi r = base_epi(ctx, st, fw);
+    r.kind = EPI_GATED_RES;
+    r.bias = (const float*)blk.w.at("lin2_b").p;
+    r.resid = h;
+    r.ldr = d;
+    r.gate = mod + 2 * d;
+    r.gate_step = ms;
+    enq_gemm(q, ctx->cat, ldc, blk.w.at("lin2_w"), ldc, N, (int)d, (int)(d + F), r);
+    return;
+  }
+  if (blk.type == BT_DOUBLE) {
+    const float* mi = mod;           // image stream modulation (6d)
+    const float* mt = mod + 6 * d;   // text stream modulation (6d)
+    float* h_img = h + (long)nx * d;
+    // attention half
+    enq_ln(q, h, d, ctx->xn, d, N, nx, mt, mt + d, mi, mi + d, st, fw);
+    {
+      Epi e = base_epi(ctx, st, fw);
+      enq_qkv_epi(ctx, e, nx, true);
+      e.bias = (const float*)blk.w.at("img_qkv_b").p;
+      enq_gemm(q, off_act(ctx, ctx->xn, (long)nx * d), d, blk.w.at("img_qkv_w"), d, ni, (int)(3 * d), (int)d, e);
+      Epi e2 = base_epi(ctx, st, fw);
+      enq_qkv_epi(ctx, e2, 0, true);
+      e2.bias = (const float*)blk.w.at("txt_qkv_b").p;
+      enq_gemm(q, ctx->xn, d, blk.w.at("txt_qkv_w"), d, nx, (int)(3 * d), (int)d, e2);
+    }
+    enq_attn(q, ctx->q, ctx->k, ctx->vt, ctx->vpad, ctx->cat, ldc, N, N, st, fw);
+    {
+      Epi r = base_epi(ctx, st, fw);
+      r.kind = EPI_GATED_RES;
+      r.bias = (const float*)blk.w.at("img_proj_b").p;
+      r.resid = h_img;
+      r.ldr = d;
+      r.gate = mi + 2 * d;
+      r.gate_step = ms;
+      enq_gemm(q, off_act(ctx, ctx->cat, (long)nx * ldc), ldc, blk.w.at("img_proj_w"), d, ni, (int)d, (int)d, r);
+      Epi r2 = r;
+      r2.bias = (const float*)blk.w.at("txt_proj_b").p;
+      r2.resid = h;
+      r2.gate = mt + 2 * d;
+      enq_gemm(q, ctx->cat, ldc, blk.w.at("txt_proj_w"), d, nx, (int)d, (int)d, r2);
+    }
+    // MLP half
+    enq_ln(q, h, d, ctx->xn, d, N, nx, mt + 3 * d, mt + 4 * d, mi + 3 * d, mi + 4 * d, st, fw);
+    {
+      Epi u = base_epi(ctx, st, fw);
+      u.kind = EPI_GELU;
+      u.out_bf16 = ctx->act_bf16;
+      u.ldo = ldc;
+      u.bias = (const float*)blk.w.at("img_up_b").p;
+      u.out = off_act(ctx, ctx->cat, (long)nx * ldc + d);
+      enq_gemm(q, off_act(ctx, ctx->xn, (long)nx * d), d, blk.w.at("img_up_w"), d, ni, (int)F, (int)d, u);
+      Epi u2 = u;
+      u2.bias = (const float*)blk.w.at("txt_up_b").p;
+      u2.out = off_act(ctx, ctx->cat, d);
+      enq_gemm(q, ctx->xn, d, blk.w.at("txt_up_w"), d, nx, (int)F, (int)d, u2);
+      Epi r = base_epi(ctx, st, fw);
+      r.kind = EPI_GATED_RES;
+      r.bias = (const float*)blk.w.at("img_down_b").p;
+      r.resid = h_img;
+      r.ldr = d;
+      r.gate = mi + 5 * d;
+      r.gate_step = ms;
+      enq_gemm(q, off_act(ctx, ctx->cat, (long)nx * ldc + d), ldc, blk.w.at("img_down_w"), F, ni, (int)d, (int)F, r);
+      Epi r2 = r;
+      r2.bias = (const float*)blk.w.at("txt_down_b").p;
+      r2.resid = h;
+      r2.gate = mt + 5 * d;
+      enq_gemm(q, off_act(ctx, ctx->cat, d), ldc, blk.w.at("txt_down_w"), F, nx, (int)d, (int)F, r2);
+    }
+    return;
+  }
+  // Wan block: self-attention, cross-attention, FFN
+  enq_ln(q, h, d, ctx->xn, d, ni, 0, mod, mod + d, mod, mod + d, st, fw);
+  {
+    Epi e = base_epi(ctx, st, fw);
+    enq_qkv_epi(ctx, e, 0, true);
+    e.bias = (const float*)blk.w.at("sa_qkv_b").p;
+    enq_gemm(q, ctx->xn, d, blk.w.at("sa_qkv_w"), d, ni, (int)(3 * d), (int)d, e);
+  }
+  enq_attn(q, ctx->q, ctx->k, ctx->vt, ctx->vpad, ctx->cat, ldc, ni, ni, st, fw);
+  {
+    Epi r = base_epi(ctx, st, fw);
+    r.kind = EPI_GATED_RES;
+    r.bias = (const float*)blk.w.at("sa_o_b").p;
+    r.resid = h;
+    r.ldr = d;
+    r.gate = mod + 2 * d;
+    r.gate_step = ms;
+    enq_gemm(q, ctx->cat, ldc, blk.w.at("sa_o_w"), d, ni, (int)d, (int)d, r);
+  }
+  enq_ln(q, h, d, ctx->xn, d, ni, 0, nullptr, nullptr, nullptr, nullptr, st, fw);
+  {
+    Epi e = base_epi(ctx, st, fw);
+    e.kind = EPI_STORE;
+    e.out = ctx->qc;
+    e.ldo = d;
+    e.out_bf16 = ctx->act_bf16;
+    e.bias = (const float*)blk.w.at("ca_q_b").p;
+    enq_gemm(q, ctx->xn, d, blk.w.at("ca_q_w"), d, ni, (int)d, (int)d, e);
+    Epi kv = base_epi(ctx, st, fw);
+    kv.kind = EPI_QKV;
+    kv.q = nullptr;
+    kv.k = ctx->kc;
+    kv.v = ctx->vtc;
+    kv.v_mode = ctx->act_bf16 ? 1 : 0;
+    kv.vpad = ctx->vpad_c;
+    kv.ldqk = d;
+    kv.d = (int)d;
+    kv.dh = ctx->dh;
+    kv.row_off = 0;
+    kv.col_base = (int)d;
+    kv.rope = nullptr;
+    kv.bias = (const float*)blk.w.at("ca_kv_b").p;
+    enq_gemm(q, ctx->txt_stage, d, blk.w.at("ca_kv_w"), d, nx, (int)(2 * d), (int)d, kv);
+  }
+  enq_attn(q, ctx->qc, ctx->kc, ctx->vtc, ctx->vpad_c, ctx->cat, ldc, ni, nx, st, fw);
+  {
+    Epi r = base_epi(ctx, st, fw);
+    r.kind = EPI_RES_ADD;
+    r.bias = (const float*)blk.w.at("ca_o_b").p;
+    r.resid = h;
+    r.ldr = d;
+    enq_gemm(q, ctx->cat, ldc, blk.w.at("ca_o_w"), d, ni, (int)d, (int)d, r);
+  }
+  enq_ln(q, h, d, ctx->xn, d, ni, 0, mod + 3 * d, mod + 4 * d, mod + 3 * d, mod + 4 * d, st, fw);
+  {
+    Epi u = base_epi(ctx, st, fw);
+    u.kind = EPI_GELU;
+    u.out_bf16 = ctx->act_bf16;
+    u.ldo = ldc;
+    u.bias = (const float*)blk.w.at("ffn_up_b").p;
+    u.out = off_act(ctx, ctx->cat, d);
+    enq_gemm(q, ctx->xn, d, blk.w.at("ffn_up_w"), d, ni, (int)F, (int)d, u);
+    Epi r = base_epi(ctx, st, fw);
+    r.kind = EPI_GATED_RES;
+    r.bias = (const float*)blk.w.at("ffn_down_b").p;
+    r.resid = h;
+    r.ldr = d;
+    r.gate = mod + 5 * d;
+    r.gate_step = ms;
+    enq_gemm(q, off_act(ctx, ctx->cat, d), ldc, blk.w.at("ffn_down_w"), F, ni, (int)d, (int)F, r);
+  }
+}
+
+static float* img_stream(bag_ctx* ctx) {
+  return ctx->arch.kind == BAG_KIND_WAN ? ctx->hj : ctx->hj + (long)ctx->nx * ctx->d;
+}
+
+static void enq_prefix(Enq& q, int use_cond, unsigned long long handle) {
+  bag_ctx* ctx = q.ctx;
+  const long d = ctx->d;
+  Epi pe = base_epi(ctx, ctx->st, -1);
+  pe.kind = EPI_DUAL_F32;
+  pe.bias = (const float*)ctx->G.at("pe_b").p;
+  pe.out = ctx->h_in;
+  pe.ldo = d;
+  pe.out2 = img_stream(ctx);
+  pe.ldo2 = d;
+  enq_gemm(q, ctx->act_bf16 ? (const void*)ctx->xb : (const void*)ctx->x, ctx->C, ctx->G.at("pe_w"),
+           ctx->C, ctx->ni, (int)d, ctx->C, pe);
+  // signal: block 0's first modulated input on the image stream (Eq. 3 drift)
+  const Block& b0 = ctx->blocks[0];
+  const float* m0 = ctx->mod_all + b0.mod_off;  // image-stream modulation comes first
+  LnArgs a{};
+  a.x = ctx->h_in;
+  a.ldx = d;
+  a.y = ctx->m_cur;
+  a.ldy = d;
+  a.y_bf16 = ctx->act_bf16;
+  a.rows = ctx->ni;
+  a.cols = (int)d;
+  a.split = 0;
+  a.shift_a = a.shift_b = m0;
+  a.scale_a = a.scale_b = m0 + d;
+  a.mod_step = ctx->mod_stride;
+  a.sig_ref = ctx->m_last;
+  a.sig_partial = ctx->sig_partial;
+  a.sig_on = 1;
+  a.st = ctx->st;
+  a.flag_want = -1;
+  q.chk(ln_mod(a, q.s));
+  q.chk(gate_step(ctx->st, ctx->sig_partial, ctx->ni, ctx->d_gate, ctx->thr, ctx->T, ctx->B,
+                  ctx->policy, ctx->d_pmask, ctx->log, handle, use_cond, q.s));
+}
+
+static void enq_full(Enq& q, int fw) {
+  bag_ctx* ctx = q.ctx;
+  const long d = ctx->d;
+  if (ctx->arch.kind != BAG_KIND_WAN)
+    q.chk(copy_rows_f32(ctx->st, fw, ctx->hj, d, ctx->txt_stage, d, ctx->act_bf16, ctx->nx, (int)d, q.s));
+  for (int b = 0; b < ctx->nblk; ++b) enq_block(q, b, ctx->hj, ctx->st, fw);
+  q.chk(cache_refresh(ctx->st, img_stream(ctx), ctx->h_in, ctx->R, ctx->m_last, ctx->m_cur,
+                      (long)ctx->ni * d, (long)ctx->ni * d, ctx->act_bf16, fw, q.s));
+}
+
+static void enq_skip(Enq& q, int fw) {
+  bag_ctx* ctx = q.ctx;
+  q.chk(cache_reuse(ctx->st, img_stream(ctx), ctx->h_in, ctx->R, (long)ctx->ni * ctx->d, fw, q.s));
+}
+
+static void enq_suffix(Enq& q) {
+  bag_ctx* ctx = q.ctx;
+  const long d = ctx->d;
+  const float* fm = ctx->mod_all + ctx->fmod_off;
+  enq_ln(q, img_stream(ctx), d, ctx->xn, d, ctx->ni, 0, fm, fm + d, fm, fm + d, ctx->st, -1);
+  Epi e = base_epi(ctx, ctx->st, -1);
+  e.kind = EPI_EULER;
+  e.bias = (const float*)ctx->G.at("fin_b").p;
+  e.x = ctx->x;
+  e.xb = ctx->act_bf16 ? ctx->xb : nullptr;
+  e.ldx = ctx->C;
+  e.dsig = ctx->dsig;
+  enq_gemm(q, ctx->xn, d, ctx->G.at("fin_w"), d, ctx->ni, ctx->C, (int)d, e);
+  q.chk(advance_step(ctx->st, q.s));
+}
+
+// Per-sample conditioning: time embedding and every modulation vector for all T steps
+// in three GEMMs (the modulation weights are read once per sample).
+static bag_status enq_prepare(bag_ctx* ctx, const bag_cond* cond) {
+  if (!cond || !cond->txt) return fail(ctx, BAG_EINVAL, "cond->txt is null");
+  if (ctx->arch.kind != BAG_KIND_WAN && !cond->pooled) return fail(ctx, BAG_EINVAL, "cond->pooled is null");
+  const long d = ctx->d;
+  cudaStream_t s = ctx->stream;
+  if (cond->txt != ctx->txt_stage)
+    CK(cudaMemcpyAsync(ctx->txt_stage, cond->txt, (size_t)ctx->nx * d * ctx->act_size, cudaMemcpyDeviceToDevice, s));
+  if (ctx->arch.kind != BAG_KIND_WAN && cond->pooled != ctx->pooled_stage)
+    CK(cudaMemcpyAsync(ctx->pooled_stage, cond->pooled, (size_t)d * 4, cudaMemcpyDeviceToDevice, s));
+  long cnt = 0;
+  Enq q{ctx, s, &cnt};
+  q.chk(sinusoid_all(ctx->sin_all, ctx->act_bf16, ctx->T, kTembDim, s));
+  Epi e1 = base_epi(ctx, nullptr, -1);
+  e1.kind = EPI_SILU;
+  e1.bias = (const float*)ctx->G.at("t1_b").p;
+  e1.out = ctx->t1o;
+  e1.ldo = d;
+  e1.out_bf16 = ctx->act_bf16;
+  enq_gemm(q, ctx->sin_all, kTembDim, ctx->G.at("t1_w"), kTembDim, ctx->T, (int)d, kTembDim, e1);
+  Epi e2 = base_epi(ctx, nullptr, -1);
+  e2.kind = EPI_VEC;
+  e2.bias = (const float*)ctx->G.at("t2_b").p;
+  e2.out = ctx->vec_all;
+  e2.ldo = d;
+  e2.addend = ctx->arch.kind == BAG_KIND_WAN ? nullptr : ctx->pooled_stage;
+  e2.out2 = ctx->svec;
+  e2.ldo2 = d;
+  e2.out2_bf16 = ctx->act_bf16;
+  enq_gemm(q, ctx->t1o, d, ctx->G.at("t2_w"), d, ctx->T, (int)d, (int)d, e2);
+  Epi e3 = base_epi(ctx, nullptr, -1);
+  e3.kind = EPI_STORE;
+  e3.bias = ctx->bmod;
+  e3.out_bf16 = 0;
+  if (ctx->arch.kind == BAG_KIND_WAN) {
+    e3.out = ctx->wan_shared;
+    e3.ldo = 8 * d;
+    enq_gemm(q, ctx->svec, d, ctx->wmod, d, ctx->T, (int)ctx->n_mod, (int)d, e3);
+    q.chk(expand_wan_mod(ctx->mod_all, ctx->wan_shared, ctx->wan_tabs, ctx->T, ctx->nblk, (int)d, s));
+  } else {
+    e3.out = ctx->mod_all;
+    e3.ldo = ctx->mod_stride;
+    enq_gemm(q, ctx->svec, d, ctx->wmod, d, ctx->T, (int)ctx->n_mod, (int)d, e3);
+  }
+  if (q.e != cudaSuccess) return fail(ctx, BAG_ECUDA, std::string("prepare: ") + cudaGetErrorString(q.e));
+  ctx->n_prepare = cnt;
+  ctx->prepared = true;
+  return BAG_OK;
+}
+
+static void destroy_graph(bag_ctx* ctx) {
+  if (ctx->exec) cudaGraphExecDestroy(ctx->exec);
+  if (ctx->graph) cudaGraphDestroy(ctx->graph);
+  ctx->exec = nullptr;
+  ctx->graph = nullptr;
+}
+
+// Capture one step: prefix, conditional node (body 0: full network; body 1: reuse),
+// suffix.  The gate kernel sets the condition on the device.
+static bag_status build_graph(bag_ctx* ctx) {
+  destroy_graph(ctx);
+  cudaStream_t s = ctx->stream;
+  if (!ctx->cap_stream) CK(cudaStreamCreateWithFlags(&ctx->cap_stream, cudaStreamNonBlocking));
+  CK(cudaGraphCreate(&ctx->graph, 0));
+  cudaGraphConditionalHandle handle;
+  CK(cudaGraphConditionalHandleCreate(&handle, ctx->graph, 0, 0));
+  CK(cudaStreamBeginCaptureToGraph(s, ctx->graph, nullptr, nullptr, 0, cudaStreamCaptureModeThreadLocal));
+  long cnt = 0;
+  Enq q{ctx, s, &cnt};
+  enq_prefix(q, 1, (unsigned long long)handle);
+  ctx->n_prefix = cnt;
+  cudaStreamCaptureStatus cs;
+  const cudaGraphNode_t* deps = nullptr;
+  size_t ndeps = 0;
+  cudaGraph_t cg = nullptr;
+  cudaError_t e = cudaStreamGetCaptureInfo(s, &cs, nullptr, &cg, &deps, nullptr, &ndeps);
+  cudaGraphNode_t cnode = nullptr;
+  cudaGraphNodeParams p = {};
+  if (e == cudaSuccess && q.e == cudaSuccess) {
+    p.type = cudaGraphNodeTypeConditional;
+    p.conditional.handle = handle;
+    p.conditional.type = cudaGraphCondTypeIf;
+    p.conditional.size = 2;
+    e = cudaGraphAddNode(&cnode, cg, deps, nullptr, ndeps, &p);
+  }
+  if (e == cudaSuccess) e = cudaStreamUpdateCaptureDependencies(s, &cnode, nullptr, 1, cudaStreamSetCaptureDependencies);
+  if (e == cudaSuccess) {
+    cudaGraph_t bodies[2] = {p.conditional.phGraph_out[0], p.conditional.phGraph_out[1]};
+    for (int bi = 0; bi < 2 && e == cudaSuccess; ++bi) {
+      e = cudaStreamBeginCaptureToGraph(ctx->cap_stream, bodies[bi], nullptr, nullptr, 0,
+                                        cudaStreamCaptureModeThreadLocal);
+      if (e != cudaSuccess) break;
+      long c2 = 0;
+      Enq qb{ctx, ctx->cap_stream, &c2};
+      if (bi == 0)
+        enq_full(qb, 1);
+      else
+        enq_skip(qb, 0);
+      cudaGraph_t tmp;
+      cudaError_t e2 = cudaStreamEndCapture(ctx->cap_stream, &tmp);
+      if (qb.e != cudaSuccess) e = qb.e;
+      if (e2 != cudaSuccess && e == cudaSuccess) e = e2;
+      if (bi == 0)
+        ctx->n_full = c2;
+      else
+        ctx->n_skip = c2;
+    }
+  }
+  cnt = 0;
+  if (e == cudaSuccess) {
+    Enq qs{ctx, s, &cnt};
+    enq_suffix(qs);
+    e = qs.e;
+  }
+  ctx->n_suffix = cnt;
+  cudaGraph_t out = nullptr;
+  cudaError_t e3 = cudaStreamEndCapture(s, &out);
+  if (e == cudaSuccess) e = e3;
+  if (e == cudaSuccess) e = cudaGraphInstantiate(&ctx->exec, ctx->graph, 0);
+  if (e != cudaSuccess) {
+    destroy_graph(ctx);
+    cudaGetLastError();
+    return fail(ctx, BAG_ECUDA, std::string("step graph capture: ") + cudaGetErrorString(e));
+  }
+  return BAG_OK;
+}
+
+// Enqueue one step.  Graph mode replays the captured step; direct mode launches every
+// kernel and the two bodies' kernels skip themselves on the device flag.
+static bag_status launch_step(bag_ctx* ctx) {
+  if (ctx->use_graph) {
+    if (!ctx->exec) CKS(build_graph(ctx));
+    CK(cudaGraphLaunch(ctx->exec, ctx->stream));
+    return BAG_OK;
+  }
+  long cnt = 0;
+  Enq q{ctx, ctx->stream, &cnt};
+  enq_prefix(q, 0, 0);
+  enq_full(q, 1);
+  enq_skip(q, 0);
+  enq_suffix(q);
+  if (q.e != cudaSuccess) return fail(ctx, BAG_ECUDA, std::string("step: ") + cudaGetErrorString(q.e));
+  return BAG_OK;
+}
+
+static bag_status check_device_error(bag_ctx* ctx) {
+  DevState h;
+  CK(cudaMemcpyAsync(&h, ctx->st, sizeof(h), cudaMemcpyDeviceToHost, ctx->stream));
+  CK(cudaStreamSynchronize(ctx->stream));
+  if (h.err) return fail(ctx, BAG_EDEVICE_TIMEOUT, "a kernel's bounded wait expired");
+  return BAG_OK;
+}
+
+static bag_status reset_state(bag_ctx* ctx) {
+  DevState h{};
+  h.t = 0;
+  h.c = 0;
+  h.t_last = -1;
+  CK(cudaMemcpyAsync(ctx->st, &h, sizeof(h), cudaMemcpyHostToDevice, ctx->stream));
+  ctx->next_t = 0;
+  ctx->prepared = false;
+  return BAG_OK;
+}
+
+// Order the internal stream after the caller's stream, and the caller's stream after
+// the work just enqueued.
+static bag_status enter(bag_ctx* ctx) {
+  CK(cudaEventRecord(ctx->ev_in, ctx->user_stream));
+  CK(cudaStreamWaitEvent(ctx->stream, ctx->ev_in, 0));
+  return BAG_OK;
+}
+static bag_status leave(bag_ctx* ctx, bag_status s) {
+  if (cudaEventRecord(ctx->ev_out, ctx->stream) == cudaSuccess)
+    cudaStreamWaitEvent(ctx->user_stream, ctx->ev_out, 0);
+  return s;
+}
+
+// ---------------------------------------------------------------------------
+// C ABI
+// ---------------------------------------------------------------------------
+static bag_status bag_reset_impl(bag_ctx* ctx) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(reset_state(ctx));
+  return BAG_OK;
+}
+
+static bag_status bag_prepare_impl(bag_ctx* ctx, const bag_cond* cond) {
+  if (!ctx) return BAG_EINVAL;
+  return enq_prepare(ctx, cond);
+}
+
+static bag_status bag_step_impl(bag_ctx* ctx, const float* x, int t, const bag_cond* cond, float* x_out,
+                    int32_t* full_or_cached) {
+  if (!ctx) return BAG_EINVAL;
+  if (!x || !x_out) return fail(ctx, BAG_EINVAL, "x / x_out is null");
+  if (t != ctx->next_t || t >= ctx->T)
+    return fail(ctx, BAG_EORDER, "step " + std::to_string(t) + " called, expected " + std::to_string(ctx->next_t));
+  if (t == 0) CKS(enq_prepare(ctx, cond));
+  if (!ctx->prepared) return fail(ctx, BAG_ESTATE, "sample not prepared");
+  const size_t xbytes = (size_t)ctx->ni * ctx->C * 4;
+  CK(cudaMemcpyAsync(ctx->x, x, xbytes, cudaMemcpyDeviceToDevice, ctx->stream));
+  if (ctx->act_bf16) CK(to_bf16(ctx->xb, ctx->x, (long)ctx->ni * ctx->C, ctx->stream));
+  CKS(launch_step(ctx));
+  CK(cudaMemcpyAsync(x_out, ctx->x, xbytes, cudaMemcpyDeviceToDevice, ctx->stream));
+  if (full_or_cached)
+    CK(cudaMemcpyAsync(full_or_cached, &ctx->st->flag, 4, cudaMemcpyDeviceToDevice, ctx->stream));
+  ctx->next_t++;
+  return BAG_OK;
+}
+
+static bag_status bag_run_impl(bag_ctx* ctx, float* x_inout, const bag_cond* cond, bag_stats* stats) {
+  if (!ctx) return BAG_EINVAL;
+  if (!x_inout) return fail(ctx, BAG_EINVAL, "x is null");
+  if (ctx->next_t != 0) return fail(ctx, BAG_ESTATE, "bag_run needs a fresh sample (bag_reset)");
+  CKS(enq_prepare(ctx, cond));
+  const size_t xbytes = (size_t)ctx->ni * ctx->C * 4;
+  CK(cudaMemcpyAsync(ctx->x, x_inout, xbytes, cudaMemcpyDeviceToDevice, ctx->stream));
+  if (ctx->act_bf16) CK(to_bf16(ctx->xb, ctx->x, (long)ctx->ni * ctx->C, ctx->stream));
+  for (int t = 0; t < ctx->T; ++t) CKS(launch_step(ctx));
+  CK(cudaMemcpyAsync(x_inout, ctx->x, xbytes, cudaMemcpyDeviceToDevice, ctx->stream));
+  ctx->next_t = ctx->T;
+  DevState h;
+  CK(cudaMemcpyAsync(&h, ctx->st, sizeof(h), cudaMemcpyDeviceToHost, ctx->stream));
+  std::vector<float> lg;
+  if (stats) {
+    lg.resize((size_t)ctx->T * kLogFloats);
+    CK(cudaMemcpyAsync(lg.data(), ctx->log, lg.size() * 4, cudaMemcpyDeviceToHost, ctx->stream));
+  }
+  CK(cudaStreamSynchronize(ctx->stream));
+  const long per_step = ctx->n_prefix + ctx->n_suffix;
+  ctx->launches = ctx->n_prepare + 2 + (long)ctx->T * per_step + (long)h.c * ctx->n_full +
+                  (long)(ctx->T - h.c) * ctx->n_skip;
+  if (stats) {
+    stats->T = ctx->T;
+    stats->B = ctx->B;
+    stats->nfe = h.c;
+    if (stats->mask)
+      for (int t = 0; t < ctx->T; ++t) stats->mask[t] = lg[(size_t)t * kLogFloats + 5] != 0.f;
+    if (stats->log) std::memcpy(stats->log, lg.data(), lg.size() * 4);
+  }
+  if (h.err) return fail(ctx, BAG_EDEVICE_TIMEOUT, "a kernel's bounded wait expired");
+  return BAG_OK;
+}
+
+static bag_status bag_run_host_impl(bag_ctx* ctx, float* x_host, const float* txt_host, const float* pooled_host,
+                        bag_stats* stats) {
+  if (!ctx) return BAG_EINVAL;
+  if (!x_host || !txt_host) return fail(ctx, BAG_EINVAL, "host buffer is null");
+  if (ctx->arch.kind != BAG_KIND_WAN && !pooled_host) return fail(ctx, BAG_EINVAL, "pooled is null");
+  if (ctx->next_t != 0) return fail(ctx, BAG_ESTATE, "bag_run_host needs a fresh sample (bag_reset)");
+  const long d = ctx->d;
+  const size_t xbytes = (size_t)ctx->ni * ctx->C * 4;
+  // stage: latent into the working buffer, text (fp32) into the scratch then convert
+  CK(cudaMemcpyAsync(ctx->x, x_host, xbytes, cudaMemcpyHostToDevice, ctx->stream));
+  CK(cudaMemcpyAsync(ctx->tmp_f32, txt_host, (size_t)ctx->nx * d * 4, cudaMemcpyHostToDevice, ctx->stream));
+  if (pooled_host) CK(cudaMemcpyAsync(ctx->pooled_stage, pooled_host, (size_t)d * 4, cudaMemcpyHostToDevice, ctx->stream));
+  void* txt_dev = ctx->txt_stage;
+  if (ctx->act_bf16)
+    CK(to_bf16((__nv_bfloat16*)ctx->txt_stage, ctx->tmp_f32, (long)ctx->nx * d, ctx->stream));
+  else
+    CK(cudaMemcpyAsync(ctx->txt_stage, ctx->tmp_f32, (size_t)ctx->nx * d * 4, cudaMemcpyDeviceToDevice, ctx->stream));
+  bag_cond cond{txt_dev, ctx->pooled_stage};
+  if (ctx->arch.kind == BAG_KIND_WAN) cond.pooled = nullptr;
+  CKS(bag_run_impl(ctx, ctx->x, &cond, stats));
+  CK(cudaMemcpyAsync(x_host, ctx->x, xbytes, cudaMemcpyDeviceToHost, ctx->stream));
+  CK(cudaStreamSynchronize(ctx->stream));
+  return BAG_OK;
+}
+
+static bag_status bag_forward_block_impl(bag_ctx* ctx, int block, int t_mod, float* h) {
+  if (!ctx || !h) return BAG_EINVAL;
+  if (block < 0 || block >= ctx->nblk) return fail(ctx, BAG_EINVAL, "block out of range");
+  if (t_mod < 0 || t_mod >= ctx->T) return fail(ctx, BAG_EINVAL, "t_mod out of range");
+  if (!ctx->prepared) return fail(ctx, BAG_ESTATE, "call bag_prepare first");
+  DevState hs{};
+  hs.t = t_mod;
+  hs.flag = 1;
+  CK(cudaMemcpyAsync(ctx->st_op, &hs, sizeof(hs), cudaMemcpyHostToDevice, ctx->stream));
+  long cnt = 0;
+  Enq q{ctx, ctx->stream, &cnt};
+  enq_block(q, block, h, ctx->st_op, -1);
+  if (q.e != cudaSuccess) return fail(ctx, BAG_ECUDA, std::string("block: ") + cudaGetErrorString(q.e));
+  ctx->launches = cnt;
+  return BAG_OK;
+}
+
+static bag_status bag_gemm_bf16_impl(bag_ctx* ctx, const void* A, long lda, const void* W, long ldw,
+                         const float* bias, float* C, long ldc, int M, int N, int K, int epilogue,
+                         int force_simt) {
+  if (!ctx || !A || !W || !C) return BAG_EINVAL;
+  if (M < 0 || N <= 0 || K <= 0 || N % 64 || K % 64 || lda < K || ldw < K || ldc < N)
+    return fail(ctx, BAG_EINVAL, "bad gemm shape");
+  Epi e;
+  e.kind = epilogue == 1 ? EPI_GELU : EPI_STORE;
+  e.bias = bias;
+  e.out = C;
+  e.ldo = ldc;
+  e.out_bf16 = 0;
+  CK(gemm(A, lda, W, ldw, M, N, K, 1, e, &ctx->st_op->err, ctx->stream, force_simt));
+  return BAG_OK;
+}
+
+static bag_status bag_attention_bf16_impl(bag_ctx* ctx, const void* q, const void* k, const void* v, void* o,
+                              long ld, int nq, int nk, int heads, int dh, int force_simt) {
+  if (!ctx || !q || !k || !v || !o) return BAG_EINVAL;
+  if (nq < 0 || nk <= 0 || heads <= 0 || (dh != 64 && dh != 128) || ld < (long)heads * dh)
+    return fail(ctx, BAG_EINVAL, "bad attention shape");
+  AttnArgs a{};
+  a.q = q;
+  a.ldq = ld;
+  a.k = k;
+  a.ldk = ld;
+  a.v = v;
+  a.v_mode = 0;
+  a.ldv = ld;
+  a.o = o;
+  a.ldo = ld;
+  a.nq = nq;
+  a.nk = nk;
+  a.heads = heads;
+  a.dh = dh;
+  a.bf16 = 1;
+  a.st = nullptr;
+  a.flag_want = -1;
+  CK(attention(a, &ctx->st_op->err, ctx->stream, force_simt));
+  return BAG_OK;
+}
+
+static bag_status bag_ln_mod_impl(bag_ctx* ctx, const float* x, const float* shift, const float* scale, void* y,
+                      int rows, int cols) {
+  if (!ctx || !x || !y) return BAG_EINVAL;
+  if (rows < 0 || cols <= 0 || cols % 4) return fail(ctx, BAG_EINVAL, "bad ln shape");
+  LnArgs a{};
+  a.x = x;
+  a.ldx = cols;
+  a.y = y;
+  a.ldy = cols;
+  a.y_bf16 = 1;
+  a.rows = rows;
+  a.cols = cols;
+  a.split = 0;
+  a.shift_a = a.shift_b = shift;
+  a.scale_a = a.scale_b = scale;
+  a.mod_step = 0;
+  a.flag_want = -1;
+  CK(ln_mod(a, ctx->stream));
+  return BAG_OK;
+}
+
+static bag_status bag_residual_add_impl(bag_ctx* ctx, float* out, const float* h_in, const float* R, long n) {
+  if (!ctx || !out || !h_in || !R) return BAG_EINVAL;
+  if (n < 0 || n % 4) return fail(ctx, BAG_EINVAL, "n must be a multiple of 4");
+  CK(residual_add(out, h_in, R, n, ctx->stream));
+  return BAG_OK;
+}
+
+extern "C" {
+
+bag_status bag_create(const bag_arch* arch, int T, int B, bag_ctx** out) {
+  if (!out) return fail(nullptr, BAG_EINVAL, "out is null");
+  *out = nullptr;
+  CKS(validate_arch(arch, T, B));
+  bag_ctx* ctx = new bag_ctx();
+  ctx->arch = *arch;
+  ctx->T = T;
+  ctx->B = B;
+  ctx->d = arch->hidden;
+  ctx->H = arch->heads;
+  ctx->dh = arch->hidden / arch->heads;
+  ctx->F = arch->mlp;
+  ctx->C = arch->patch_ch;
+  ctx->ni = arch->grid[0] * arch->grid[1] * arch->grid[2];
+  ctx->nx = arch->n_txt;
+  ctx->N = ctx->ni + ctx->nx;
+  ctx->nrope = arch->kind == BAG_KIND_WAN ? ctx->ni : ctx->N;
+  ctx->act_bf16 = arch->dtype == BAG_BF16;
+  ctx->act_size = ctx->act_bf16 ? 2 : 4;
+  ctx->thr = (float)std::log((double)arch->tau / (1.0 - (double)arch->tau));
+  if (arch->kind == BAG_KIND_WAN) {
+    ctx->nblk = arch->n_wan;
+    ctx->blocks.assign(ctx->nblk, Block{});
+    for (auto& b : ctx->blocks) b.type = BT_WAN;
+  } else {
+    ctx->nblk = arch->n_double + arch->n_single;
+    ctx->blocks.assign(ctx->nblk, Block{});
+    for (int i = 0; i < ctx->nblk; ++i) ctx->blocks[i].type = i < arch->n_double ? BT_DOUBLE : BT_SINGLE;
+  }
+  bag_status s = BAG_OK;
+  if (cudaStreamCreateWithFlags(&ctx->stream, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ctx->ev_in, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ctx->ev_out, cudaEventDisableTiming) != cudaSuccess)
+    s = fail(ctx, BAG_ECUDA, "stream/event creation failed");
+  if (s == BAG_OK && kernels_init() != cudaSuccess) s = fail(ctx, BAG_ECUDA, "kernel attribute setup failed");
+  if (s == BAG_OK) s = alloc_weights(ctx);
+  if (s == BAG_OK) s = alloc_activations(ctx);
+  if (s == BAG_OK) s = seed_weights(ctx);
+  if (s == BAG_OK) s = seed_gate(ctx);
+  if (s == BAG_OK) s = reset_state(ctx);
+  if (s == BAG_OK && cudaStreamSynchronize(ctx->stream) != cudaSuccess) s = fail(ctx, BAG_ECUDA, "create sync failed");
+  if (s != BAG_OK) {
+    g_create_error = ctx->err;
+    bag_destroy(ctx);
+    return s;
+  }
+  *out = ctx;
+  return BAG_OK;
+}
+
+void bag_destroy(bag_ctx* ctx) {
+  if (!ctx) return;
+  destroy_graph(ctx);
+  if (ctx->cap_stream) cudaStreamDestroy(ctx->cap_stream);
+  if (ctx->warena) cudaFree(ctx->warena);
+  if (ctx->aarena) cudaFree(ctx->aarena);
+  if (ctx->ev_in) cudaEventDestroy(ctx->ev_in);
+  if (ctx->ev_out) cudaEventDestroy(ctx->ev_out);
+  if (ctx->stream) cudaStreamDestroy(ctx->stream);
+  delete ctx;
+}
+
+const char* bag_last_error(bag_ctx* ctx) { return ctx ? ctx->err.c_str() : g_create_error.c_str(); }
+
+bag_status bag_set_stream(bag_ctx* ctx, void* stream) {
+  if (!ctx) return BAG_EINVAL;
+  ctx->user_stream = (cudaStream_t)stream;
+  return BAG_OK;
+}
+
+bag_status bag_load_gate(bag_ctx* ctx, const float* theta, const float* mu, const float* sd) {
+  if (!ctx) return BAG_EINVAL;
+  if (!theta) return fail(ctx, BAG_EINVAL, "theta is null");
+  float g[kGateFloats];
+  std::memcpy(g, theta, 81 * sizeof(float));
+  for (int i = 0; i < 3; ++i) {
+    g[81 + i] = mu ? mu[i] : 0.f;
+    g[84 + i] = sd ? sd[i] : 1.f;
+    if (!(g[84 + i] != 0.f)) return fail(ctx, BAG_EINVAL, "sd must be nonzero");
+  }
+  CK(cudaMemcpyAsync(ctx->d_gate, g, sizeof(g), cudaMemcpyHostToDevice, ctx->stream));
+  CK(cudaStreamSynchronize(ctx->stream));
+  return BAG_OK;
+}
+
+bag_status bag_set_policy(bag_ctx* ctx, int policy, const uint8_t* host_mask) {
+  if (!ctx) return BAG_EINVAL;
+  if (policy < 0 || policy > 2) return fail(ctx, BAG_EINVAL, "unknown policy");
+  if (policy == BAG_POLICY_MASK) {
+    if (!host_mask) return fail(ctx, BAG_EINVAL, "mask policy needs host_mask");
+    CK(cudaMemcpyAsync(ctx->d_pmask, host_mask, ctx->T, cudaMemcpyHostToDevice, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));
+  }
+  ctx->policy = policy;
+  destroy_graph(ctx);  // policy is a kernel argument of the captured gate launch
+  return BAG_OK;
+}
+
+bag_status bag_reset(bag_ctx* ctx) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, bag_reset_impl(ctx));
+}
+
+bag_status bag_prepare(bag_ctx* ctx, const bag_cond* cond) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, bag_prepare_impl(ctx, cond));
+}
+
+bag_status bag_step(bag_ctx* ctx, const float* x, int t, const bag_cond* cond, float* x_out,
+                    int32_t* full_or_cached) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, bag_step_impl(ctx, x, t, cond, x_out, full_or_cached));
+}
+
+bag_status bag_run(bag_ctx* ctx, float* x_inout, const bag_cond* cond, bag_stats* stats) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, bag_run_impl(ctx, x_inout, cond, stats));
+}
+
+bag_status bag_run_host(bag_ctx* ctx, float* x_host, const float* txt_host, const float* pooled_host,
+                        bag_stats* stats) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, bag_run_host_impl(ctx, x_host, txt_host, pooled_host, stats));
+}
+
+bag_status bag_get_weight(bag_ctx* ctx, int block, const char* name, float* out, size_t n) {
+  if (!ctx || !name || !out) return BAG_EINVAL;
+  const std::map<std::string, Tensor>* m = nullptr;
+  if (block < 0)
+    m = &ctx->G;
+  else if (block < ctx->nblk)
+    m = &ctx->blocks[block].w;
+  else
+    return fail(ctx, BAG_EINVAL, "block out of range");
+  auto it = m->find(name);
+  if (it == m->end()) return fail(ctx, BAG_EINVAL, std::string("no tensor ") + name);
+  const Tensor& t = it->second;
+  if ((long)n != t.n) return fail(ctx, BAG_EINVAL, "size mismatch: tensor has " + std::to_string(t.n));
+  if (t.bf16) {
+    std::vector<uint16_t> tmp(n);
+    CK(cudaMemcpyAsync(tmp.data(), t.p, n * 2, cudaMemcpyDeviceToHost, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));
+    for (size_t i = 0; i < n; ++i) {
+      uint32_t u = (uint32_t)tmp[i] << 16;
+      std::memcpy(out + i, &u, 4);
+    }
+  } else {
+    CK(cudaMemcpyAsync(out, t.p, n * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));
+  }
+  return BAG_OK;
+}
+
+bag_status bag_forward_block(bag_ctx* ctx, int block, int t_mod, float* h) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, bag_forward_block_impl(ctx, block, t_mod, h));
+}
+
+bag_status bag_launch_count(bag_ctx* ctx, long* out) {
+  if (!ctx || !out) return BAG_EINVAL;
+  *out = ctx->launches;
+  return BAG_OK;
+}
+
+bag_status bag_gemm_bf16(bag_ctx* ctx, const void* A, long lda, const void* W, long ldw,
+                         const float* bias, float* C, long ldc, int M, int N, int K, int epilogue,
+                         int force_simt) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, bag_gemm_bf16_impl(ctx, A, lda, W, ldw, bias, C, ldc, M, N, K, epilogue, force_simt));
+}
+
+bag_status bag_attention_bf16(bag_ctx* ctx, const void* q, const void* k, const void* v, void* o,
+                              long ld, int nq, int nk, int heads, int dh, int force_simt) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, bag_attention_bf16_impl(ctx, q, k, v, o, ld, nq, nk, heads, dh, force_simt));
+}
+
+bag_status bag_ln_mod(bag_ctx* ctx, const float* x, const float* shift, const float* scale, void* y,
+                      int rows, int cols) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, bag_ln_mod_impl(ctx, x, shift, scale, y, rows, cols));
+}
+
+bag_status bag_residual_add(bag_ctx* ctx, float* out, const float* h_in, const float* R, long n) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, bag_residual_add_impl(ctx, out, h_in, R, n));
+}
+
+}  // extern "C"

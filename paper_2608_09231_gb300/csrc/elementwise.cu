@@ -1,0 +1,450 @@
+// Memory-bound kernels of the cached denoising step and the on-device gate.
+//
+//  * ln_mod: row LayerNorm + adaLN modulation (1 + scale) * LN(x) + shift, optionally
+//    fused with the trajectory signal (per-row partial sums of |m_t - m_last| and
+//    |m_last|, the relative-L1 drift of the first block's modulated input).
+//  * gate_step: one warp; reduces the signal partials in a fixed order, forms the gate
+//    inputs, evaluates the 3->16->1 gate in fp32 with every product and sum rounded
+//    separately, applies Algorithm 2's two forced rules, updates the counters and the
+//    step log, and hands the decision to a CUDA-graph conditional node.
+//  * cache_refresh / cache_reuse: R = h_out - h_in after a full step; h_out = h_in + R
+//    on a reused step (plain residual reuse).
+//  * small helpers: step counter, sinusoidal timestep features, seeded fills.
+#include <cmath>
+
+#include "common.cuh"
+#include "epilogue.cuh"
+#include "kernels.h"
+
+namespace bag {
+
+// ---------------------------------------------------------------------------
+// LayerNorm + modulation (+ signal)
+// ---------------------------------------------------------------------------
+constexpr int LN_THREADS = 128;
+constexpr int LN_MAXV = 12;  // float4 per thread: cols <= 128 * 4 * 12 = 6144
+
+BAG_DEV float block_sum(float v, float* red) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float s = 0.f;
+#pragma unroll
+  for (int w = 0; w < LN_THREADS / 32; ++w) s += red[w];
+  return s;
+}
+
+__global__ void __launch_bounds__(LN_THREADS) ln_mod_kernel(const LnArgs a) {
+  if (epi_skip(a.st, a.flag_want)) return;
+  __shared__ float red[LN_THREADS / 32];
+  const int row = blockIdx.x;
+  if (row >= a.rows) return;
+  const int t = a.st ? a.st->t : 0;
+  const float* x = a.x + (long)row * a.ldx;
+  const int nv = a.cols / 4;
+  float4 v[LN_MAXV];
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < LN_MAXV; ++i) {
+    const int c = threadIdx.x + i * LN_THREADS;
+    if (c < nv) {
+      v[i] = reinterpret_cast<const float4*>(x)[c];
+      s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
+    }
+  }
+  const float mean = block_sum(s, red) / (float)a.cols;
+  float q = 0.f;
+#pragma unroll
+  for (int i = 0; i < LN_MAXV; ++i) {
+    const int c = threadIdx.x + i * LN_THREADS;
+    if (c < nv) {
+      const float dx = v[i].x - mean, dy = v[i].y - mean, dz = v[i].z - mean, dw = v[i].w - mean;
+      q += (dx * dx + dy * dy) + (dz * dz + dw * dw);
+    }
+  }
+  const float rstd = rsqrtf(block_sum(q, red) / (float)a.cols + 1e-6f);
+  const bool first = row < a.split;
+  const float* sh = first ? a.shift_a : a.shift_b;
+  const float* sc = first ? a.scale_a : a.scale_b;
+  if (sh) sh += (long)t * a.mod_step;
+  if (sc) sc += (long)t * a.mod_step;
+  float sig_num = 0.f, sig_den = 0.f;
+#pragma unroll
+  for (int i = 0; i < LN_MAXV; ++i) {
+    const int c = threadIdx.x + i * LN_THREADS;
+    if (c < nv) {
+      float y[4] = {(v[i].x - mean) * rstd, (v[i].y - mean) * rstd, (v[i].z - mean) * rstd,
+                    (v[i].w - mean) * rstd};
+      if (sc) {
+        const float4 s4 = reinterpret_cast<const float4*>(sc)[c];
+        y[0] *= 1.f + s4.x;
+        y[1] *= 1.f + s4.y;
+        y[2] *= 1.f + s4.z;
+        y[3] *= 1.f + s4.w;
+      }
+      if (sh) {
+        const float4 h4 = reinterpret_cast<const float4*>(sh)[c];
+        y[0] += h4.x;
+        y[1] += h4.y;
+        y[2] += h4.z;
+        y[3] += h4.w;
+      }
+      const long off = (long)row * a.ldy + 4 * c;
+      if (a.y_bf16) {
+        uint2 u;
+        u.x = pack_bf16x2(y[0], y[1]);
+        u.y = pack_bf16x2(y[2], y[3]);
+        *reinterpret_cast<uint2*>(reinterpret_cast<__nv_bfloat16*>(a.y) + off) = u;
+      } else {
+        *reinterpret_cast<float4*>(reinterpret_cast<float*>(a.y) + off) =
+            make_float4(y[0], y[1], y[2], y[3]);
+      }
+      if (a.sig_on) {
+        float r[4], yy[4];
+        if (a.y_bf16) {
+          const uint2 u = *reinterpret_cast<const uint2*>(
+              reinterpret_cast<const __nv_bfloat16*>(a.sig_ref) + off);
+          const __nv_bfloat162 r01 = *reinterpret_cast<const __nv_bfloat162*>(&u.x);
+          const __nv_bfloat162 r23 = *reinterpret_cast<const __nv_bfloat162*>(&u.y);
+          r[0] = __low2float(r01);
+          r[1] = __high2float(r01);
+          r[2] = __low2float(r23);
+          r[3] = __high2float(r23);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) yy[j] = bf16_round(y[j]);
+        } else {
+          const float4 r4 = *reinterpret_cast<const float4*>(
+              reinterpret_cast<const float*>(a.sig_ref) + off);
+          r[0] = r4.x;
+          r[1] = r4.y;
+          r[2] = r4.z;
+          r[3] = r4.w;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) yy[j] = y[j];
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          sig_num += fabsf(yy[j] - r[j]);
+          sig_den += fabsf(r[j]);
+        }
+      }
+    }
+  }
+  if (a.sig_on) {
+    const float n = block_sum(sig_num, red);
+    const float d = block_sum(sig_den, red);
+    if (threadIdx.x == 0) {
+      a.sig_partial[2 * row] = n;
+      a.sig_partial[2 * row + 1] = d;
+    }
+  }
+}
+
+cudaError_t ln_mod(const LnArgs& a, cudaStream_t s) {
+  if (a.rows <= 0) return cudaSuccess;
+  if (a.cols % 4 != 0 || a.cols > LN_THREADS * 4 * LN_MAXV) return cudaErrorInvalidValue;
+  ln_mod_kernel<<<a.rows, LN_THREADS, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+// Standalone relative-L1 partial sums (same reduction as the fused signal).
+__global__ void __launch_bounds__(LN_THREADS) rel_l1_kernel(const void* a, const void* b, int bf16,
+                                                            long cols, float* partial) {
+  __shared__ float red[LN_THREADS / 32];
+  const long row = blockIdx.x;
+  float n = 0.f, d = 0.f;
+  for (long c = threadIdx.x; c < cols; c += LN_THREADS) {
+    const long i = row * cols + c;
+    float x, y;
+    if (bf16) {
+      x = __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(a)[i]);
+      y = __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(b)[i]);
+    } else {
+      x = reinterpret_cast<const float*>(a)[i];
+      y = reinterpret_cast<const float*>(b)[i];
+    }
+    n += fabsf(x - y);
+    d += fabsf(y);
+  }
+  n = block_sum(n, red);
+  d = block_sum(d, red);
+  if (threadIdx.x == 0) {
+    partial[2 * row] = n;
+    partial[2 * row + 1] = d;
+  }
+}
+
+cudaError_t rel_l1_partials(const void* a, const void* b, int a_bf16, long rows, long cols,
+                            float* partial, cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  rel_l1_kernel<<<(unsigned)rows, LN_THREADS, 0, s>>>(a, b, a_bf16, cols, partial);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// gate + pacing (one warp)
+// ---------------------------------------------------------------------------
+// gate_params layout: w1[16][3] (row-major), b1[16], w2[16], b2, mu[3], sd[3]
+__global__ void gate_kernel(DevState* st, const float* partial, int rows, const float* gp,
+                            float thr, int T, int B, int policy, const uint8_t* pmask, float* log,
+                            cudaGraphConditionalHandle handle, int use_cond) {
+  const int lane = threadIdx.x;
+  const int t = st->t, c = st->c, t_last = st->t_last;
+  float num = 0.f, den = 0.f;
+  if (t > 0) {
+    for (int r = lane; r < rows; r += 32) {
+      num += partial[2 * r];
+      den += partial[2 * r + 1];
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      num += __shfl_xor_sync(0xffffffffu, num, off);
+      den += __shfl_xor_sync(0xffffffffu, den, off);
+    }
+  }
+  if (lane != 0) return;
+  float* L = log + (long)t * kLogFloats;
+  int m = 1, gbit = 1;
+  float z = 0.f, f0 = 0.f, f1 = 0.f, f2 = 0.f;
+  if (t > 0) {
+    f0 = __fdiv_rn((float)(B - c), (float)B);
+    f1 = __fdiv_rn((float)(T - t), (float)T);
+    f2 = __fdiv_rn(num, den);
+    const float f[3] = {f0, f1, f2};
+    float fz[3];
+#pragma unroll
+    for (int i = 0; i < 3; ++i) fz[i] = __fdiv_rn(__fsub_rn(f[i], gp[81 + i]), gp[84 + i]);
+    z = gp[80];
+    for (int j = 0; j < 16; ++j) {
+      float h = gp[48 + j];
+#pragma unroll
+      for (int i = 0; i < 3; ++i) h = __fadd_rn(h, __fmul_rn(gp[3 * j + i], fz[i]));
+      if (!(h > 0.f)) h = 0.f;
+      z = __fadd_rn(z, __fmul_rn(gp[64 + j], h));
+    }
+    gbit = z > thr ? 1 : 0;
+    if (policy == 0) {  // Algorithm 2
+      m = gbit;
+      if (B - c >= T - t) m = 1;  // spend the remainder
+      if (B - c == 0) m = 0;      // budget exhausted
+    } else if (policy == 1) {     // uncached sampling
+      m = 1;
+    } else {                      // caller-given mask
+      m = pmask[t] ? 1 : 0;
+    }
+  }
+  L[0] = f0;
+  L[1] = f1;
+  L[2] = f2;
+  L[3] = z;
+  L[4] = (float)gbit;
+  L[5] = (float)m;
+  L[6] = (float)c;
+  L[7] = t > 0 ? (float)(t - t_last) : 0.f;
+  L[8] = (float)B / (float)T;
+  L[9] = (float)(B - c) / (float)B;
+  L[10] = (float)(B - c) / (float)(T - t);
+  L[11] = num;
+  L[12] = den;
+  st->flag = m;
+  if (m) {
+    st->c = c + 1;
+    st->t_last = t;
+  }
+  if (use_cond) cudaGraphSetConditional(handle, (unsigned)m);
+}
+
+cudaError_t gate_step(DevState* st, const float* sig_partial, int sig_rows, const float* gate_params,
+                      float thr, int T, int B, int policy, const uint8_t* policy_mask, float* log,
+                      unsigned long long cond_handle, int use_cond, cudaStream_t s) {
+  gate_kernel<<<1, 32, 0, s>>>(st, sig_partial, sig_rows, gate_params, thr, T, B, policy,
+                               policy_mask, log, (cudaGraphConditionalHandle)cond_handle, use_cond);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// residual cache
+// ---------------------------------------------------------------------------
+__global__ void cache_refresh_kernel(const DevState* st, int flag_want, const float4* h_img,
+                                     const float4* h_in, float4* R, long n4, uint4* m_last,
+                                     const uint4* m_cur, long m16) {
+  if (epi_skip(st, flag_want)) return;
+  const long stride = (long)gridDim.x * blockDim.x;
+  for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
+    const float4 a = h_img[i], b = h_in[i];
+    R[i] = make_float4(a.x - b.x, a.y - b.y, a.z - b.z, a.w - b.w);
+  }
+  for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < m16; i += stride) m_last[i] = m_cur[i];
+}
+
+__global__ void cache_reuse_kernel(const DevState* st, int flag_want, float4* h_img,
+                                   const float4* h_in, const float4* R, long n4) {
+  if (epi_skip(st, flag_want)) return;
+  const long stride = (long)gridDim.x * blockDim.x;
+  for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
+    const float4 a = h_in[i], r = R[i];
+    h_img[i] = make_float4(a.x + r.x, a.y + r.y, a.z + r.z, a.w + r.w);
+  }
+}
+
+static int grid_for(long n, int threads) {
+  long b = (n + threads - 1) / threads;
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms <= 0) sms = 148;
+  }
+  long cap = (long)sms * 8;
+  if (b > cap) b = cap;
+  if (b < 1) b = 1;
+  return (int)b;
+}
+
+cudaError_t cache_refresh(const DevState* st, const float* h_img, const float* h_in, float* R,
+                          void* m_last, const void* m_cur, long n, long m_n, int m_bf16,
+                          int flag_want, cudaStream_t s) {
+  if (n % 4 != 0) return cudaErrorInvalidValue;
+  const long mbytes = m_n * (m_bf16 ? 2 : 4);
+  if (mbytes % 16 != 0) return cudaErrorInvalidValue;
+  cache_refresh_kernel<<<grid_for(n / 4, 256), 256, 0, s>>>(
+      st, flag_want, reinterpret_cast<const float4*>(h_img), reinterpret_cast<const float4*>(h_in),
+      reinterpret_cast<float4*>(R), n / 4, reinterpret_cast<uint4*>(m_last),
+      reinterpret_cast<const uint4*>(m_cur), mbytes / 16);
+  return cudaGetLastError();
+}
+
+cudaError_t cache_reuse(const DevState* st, float* h_img, const float* h_in, const float* R,
+                        long n, int flag_want, cudaStream_t s) {
+  if (n % 4 != 0) return cudaErrorInvalidValue;
+  cache_reuse_kernel<<<grid_for(n / 4, 256), 256, 0, s>>>(
+      st, flag_want, reinterpret_cast<float4*>(h_img), reinterpret_cast<const float4*>(h_in),
+      reinterpret_cast<const float4*>(R), n / 4);
+  return cudaGetLastError();
+}
+
+cudaError_t residual_add(float* out, const float* a, const float* b, long n, cudaStream_t s) {
+  return cache_reuse(nullptr, out, a, b, n, -1, s);
+}
+
+// ---------------------------------------------------------------------------
+// helpers
+// ---------------------------------------------------------------------------
+__global__ void copy_rows_kernel(const DevState* st, int flag_want, float* dst, long ldd,
+                                 const void* src, long lds, int src_bf16, int rows, int cols) {
+  if (epi_skip(st, flag_want)) return;
+  const long n = (long)rows * cols;
+  for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
+    const long r = i / cols, c = i % cols;
+    dst[r * ldd + c] = src_bf16 ? __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(src)[r * lds + c])
+                                : reinterpret_cast<const float*>(src)[r * lds + c];
+  }
+}
+
+cudaError_t copy_rows_f32(const DevState* st, int flag_want, float* dst, long ldd, const void* src,
+                          long lds, int src_bf16, int rows, int cols, cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  copy_rows_kernel<<<grid_for((long)rows * cols, 256), 256, 0, s>>>(st, flag_want, dst, ldd, src,
+                                                                    lds, src_bf16, rows, cols);
+  return cudaGetLastError();
+}
+
+__global__ void advance_kernel(DevState* st) { st->t += 1; }
+
+cudaError_t advance_step(DevState* st, cudaStream_t s) {
+  advance_kernel<<<1, 1, 0, s>>>(st);
+  return cudaGetLastError();
+}
+
+// Sinusoidal features of 1000 * sigma_t, sigma_t = 1 - t/T, for every step t < T:
+// [cos(1000 sigma_t f_j), sin(1000 sigma_t f_j)], f_j = exp(-ln(10000) j / (dim/2)).
+__global__ void sinusoid_kernel(void* out, int out_bf16, int T, int dim) {
+  const int t = blockIdx.x, j = threadIdx.x;
+  const int half = dim / 2;
+  if (t >= T || j >= dim) return;
+  const double sig = 1.0 - (double)t / (double)T;
+  const int jj = j < half ? j : j - half;
+  const double f = exp(-log(10000.0) * (double)jj / (double)half);
+  const double arg = 1000.0 * sig * f;
+  const float v = (float)(j < half ? cos(arg) : sin(arg));
+  if (out_bf16)
+    reinterpret_cast<__nv_bfloat16*>(out)[(long)t * dim + j] = __float2bfloat16_rn(v);
+  else
+    reinterpret_cast<float*>(out)[(long)t * dim + j] = v;
+}
+
+cudaError_t sinusoid_all(void* out, int out_bf16, int T, int dim, cudaStream_t s) {
+  sinusoid_kernel<<<T, dim, 0, s>>>(out, out_bf16, T, dim);
+  return cudaGetLastError();
+}
+
+// Wan: per-block modulation = shared projection of the time embedding + block table.
+// shared8d: [T][8d] (6d shared block modulation, then 2d final-layer modulation);
+// mod_all:  [T][nblocks*6d + 2d].
+__global__ void expand_wan_kernel(float* mod_all, const float* shared8d, const float* tables,
+                                  int T, int nblocks, int d) {
+  const long per = (long)nblocks * 6 * d + 2 * d;
+  const long n = (long)T * per;
+  for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
+    const long t = i / per, j = i % per;
+    const float* sh = shared8d + t * 8 * d;
+    if (j < (long)nblocks * 6 * d) {
+      const long b = j / (6 * d), c = j % (6 * d);
+      mod_all[i] = sh[c] + tables[b * 6 * d + c];
+    } else {
+      mod_all[i] = sh[6 * d + (j - (long)nblocks * 6 * d)];
+    }
+  }
+}
+
+cudaError_t expand_wan_mod(float* mod_all, const float* shared8d, const float* tables, int T,
+                           int nblocks, int d, cudaStream_t s) {
+  expand_wan_kernel<<<grid_for((long)T * nblocks * 6 * d, 256), 256, 0, s>>>(mod_all, shared8d,
+                                                                           tables, T, nblocks, d);
+  return cudaGetLastError();
+}
+
+__global__ void to_bf16_kernel(__nv_bfloat16* dst, const float* src, long n) {
+  for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x)
+    dst[i] = __float2bfloat16_rn(src[i]);
+}
+
+cudaError_t to_bf16(__nv_bfloat16* dst, const float* src, long n, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  to_bf16_kernel<<<grid_for(n, 256), 256, 0, s>>>(dst, src, n);
+  return cudaGetLastError();
+}
+
+// Seeded fill: SplitMix64 stream (state s + (i+1) * golden, finalised by mix), the four
+// 16-bit chunks summed and centred (Irwin-Hall(4)), scaled by c32 in fp32.
+BAG_DEV uint64_t sm64_mix(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__global__ void fill_synth_kernel(void* dst, long n, uint64_t start, float c32, int bf16) {
+  for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
+    const uint64_t u = sm64_mix(start + (uint64_t)(i + 1) * 0x9E3779B97F4A7C15ull);
+    const long q = (long)(u & 0xFFFF) + (long)((u >> 16) & 0xFFFF) + (long)((u >> 32) & 0xFFFF) +
+                   (long)(u >> 48) - 131070;
+    const float v = __fmul_rn((float)q, c32);
+    if (bf16)
+      reinterpret_cast<__nv_bfloat16*>(dst)[i] = __float2bfloat16_rn(v);
+    else
+      reinterpret_cast<float*>(dst)[i] = v;
+  }
+}
+
+cudaError_t fill_synth(void* dst, long n, uint64_t start, uint64_t /*unused*/, float c32, int bf16,
+                       cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  fill_synth_kernel<<<grid_for(n, 256), 256, 0, s>>>(dst, n, start, c32, bf16);
+  return cudaGetLastError();
+}
+
+}  // namespace bag

@@ -1,0 +1,177 @@
+// Fused GEMM epilogues: every projection of the DiT block finishes here, so that no
+// separate elementwise pass re-reads its output.
+//   QKV (+ RoPE on q and k, V written transposed per head for the attention kernel's
+//   K-major B operand) and the GELU'd MLP half of a single-stream block's linear1,
+//   gated residual h += g * y (out-projection, linear2, MLP down), plain/GELU/SiLU
+//   stores, and the flow-matching Euler update x += (sigma_{t+1} - sigma_t) v.
+#pragma once
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace bag {
+
+BAG_DEV int epi_step(const Epi& e) { return e.st ? e.st->t : 0; }
+
+// Early exit for kernels captured on one side of the full/reuse branch.
+BAG_DEV bool epi_skip(const DevState* st, int flag_want) {
+  return st != nullptr && flag_want >= 0 && st->flag != flag_want;
+}
+
+template <int NV>
+BAG_DEV void store_vals(void* base, long idx, const float* v, int bf16) {
+  if (bf16) {
+    __nv_bfloat16* p = reinterpret_cast<__nv_bfloat16*>(base) + idx;
+    if constexpr (NV % 8 == 0) {
+      if ((reinterpret_cast<uintptr_t>(p) & 15) == 0) {
+#pragma unroll
+        for (int j = 0; j < NV; j += 8) {
+          uint4 u;
+          u.x = pack_bf16x2(v[j], v[j + 1]);
+          u.y = pack_bf16x2(v[j + 2], v[j + 3]);
+          u.z = pack_bf16x2(v[j + 4], v[j + 5]);
+          u.w = pack_bf16x2(v[j + 6], v[j + 7]);
+          *reinterpret_cast<uint4*>(p + j) = u;
+        }
+        return;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < NV; ++j) p[j] = __float2bfloat16_rn(v[j]);
+  } else {
+    float* p = reinterpret_cast<float*>(base) + idx;
+    if constexpr (NV % 4 == 0) {
+      if ((reinterpret_cast<uintptr_t>(p) & 15) == 0) {
+#pragma unroll
+        for (int j = 0; j < NV; j += 4)
+          *reinterpret_cast<float4*>(p + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+        return;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < NV; ++j) p[j] = v[j];
+  }
+}
+
+// Apply the epilogue to NV consecutive accumulators v[0..NV) of output row `row`,
+// columns [col0, col0 + NV).  NV is even and col0 is a multiple of NV; the chunk never
+// straddles a q/k/v/mlp boundary (those are multiples of 64 columns).
+template <int NV>
+BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v) {
+  if (row >= e.M || col0 >= e.N) return;
+  if (e.bias) {
+#pragma unroll
+    for (int j = 0; j < NV; ++j) v[j] += __ldg(e.bias + col0 + j);
+  }
+  switch (e.kind) {
+    case EPI_STORE:
+      store_vals<NV>(e.out, (long)row * e.ldo + col0, v, e.out_bf16);
+      break;
+    case EPI_GELU:
+#pragma unroll
+      for (int j = 0; j < NV; ++j) v[j] = gelu_tanh(v[j]);
+      store_vals<NV>(e.out, (long)row * e.ldo + col0, v, e.out_bf16);
+      break;
+    case EPI_SILU:
+#pragma unroll
+      for (int j = 0; j < NV; ++j) v[j] = silu(v[j]);
+      store_vals<NV>(e.out, (long)row * e.ldo + col0, v, e.out_bf16);
+      break;
+    case EPI_QKV: {
+      const int lc = col0 + e.col_base;
+      const int region = lc / e.d;
+      if (region >= 3) {
+#pragma unroll
+        for (int j = 0; j < NV; ++j) v[j] = gelu_tanh(v[j]);
+        store_vals<NV>(e.mlp, (long)row * e.ldm + (lc - 3 * e.d), v, e.act_bf16);
+        break;
+      }
+      const int jr = row + e.row_off;  // joint-sequence row
+      const int cc = lc - region * e.d;
+      if (region < 2 && e.rope) {
+        const int e0 = cc % e.dh;
+        const float2* cs = e.rope + (long)jr * (e.dh / 2) + e0 / 2;
+#pragma unroll
+        for (int p = 0; p < NV / 2; ++p) {
+          const float2 r = __ldg(cs + p);
+          const float x0 = v[2 * p], x1 = v[2 * p + 1];
+          v[2 * p] = x0 * r.x - x1 * r.y;
+          v[2 * p + 1] = x0 * r.y + x1 * r.x;
+        }
+      }
+      if (region == 0) {
+        store_vals<NV>(e.q, (long)jr * e.ldqk + cc, v, e.act_bf16);
+      } else if (region == 1) {
+        store_vals<NV>(e.k, (long)jr * e.ldqk + cc, v, e.act_bf16);
+      } else if (e.v_mode == 0) {
+        store_vals<NV>(e.v, (long)jr * e.ldqk + cc, v, e.act_bf16);
+      } else {
+        // transposed per head: vt[(head * dh + e) * vpad + token]
+        if (e.act_bf16) {
+          __nv_bfloat16* vt = reinterpret_cast<__nv_bfloat16*>(e.v);
+#pragma unroll
+          for (int j = 0; j < NV; ++j) vt[(long)(cc + j) * e.vpad + jr] = __float2bfloat16_rn(v[j]);
+        } else {
+          float* vt = reinterpret_cast<float*>(e.v);
+#pragma unroll
+          for (int j = 0; j < NV; ++j) vt[(long)(cc + j) * e.vpad + jr] = v[j];
+        }
+      }
+      break;
+    }
+    case EPI_GATED_RES: {
+      const float* g = e.gate + (long)t * e.gate_step + col0;
+      float* r = e.resid + (long)row * e.ldr + col0;
+      if constexpr (NV % 4 == 0) {
+#pragma unroll
+        for (int j = 0; j < NV; j += 4) {
+          float4 h = *reinterpret_cast<float4*>(r + j);
+          h.x += __ldg(g + j) * v[j];
+          h.y += __ldg(g + j + 1) * v[j + 1];
+          h.z += __ldg(g + j + 2) * v[j + 2];
+          h.w += __ldg(g + j + 3) * v[j + 3];
+          *reinterpret_cast<float4*>(r + j) = h;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < NV; ++j) r[j] += __ldg(g + j) * v[j];
+      }
+      break;
+    }
+    case EPI_RES_ADD: {
+      float* r = e.resid + (long)row * e.ldr + col0;
+#pragma unroll
+      for (int j = 0; j < NV; ++j) r[j] += v[j];
+      break;
+    }
+    case EPI_EULER: {
+      const float ds = e.dsig[t];
+      float* x = e.x + (long)row * e.ldx + col0;
+      float nx[NV];
+#pragma unroll
+      for (int j = 0; j < NV; ++j) {
+        nx[j] = x[j] + ds * v[j];
+        x[j] = nx[j];
+      }
+      if (e.xb) store_vals<NV>(e.xb, (long)row * e.ldx + col0, nx, 1);
+      break;
+    }
+    case EPI_VEC: {
+#pragma unroll
+      for (int j = 0; j < NV; ++j) v[j] += (e.addend ? e.addend[col0 + j] : 0.f);
+      store_vals<NV>(e.out, (long)row * e.ldo + col0, v, 0);
+#pragma unroll
+      for (int j = 0; j < NV; ++j) v[j] = silu(v[j]);
+      store_vals<NV>(e.out2, (long)row * e.ldo2 + col0, v, e.out2_bf16);
+      break;
+    }
+    case EPI_DUAL_F32:
+      store_vals<NV>(e.out, (long)row * e.ldo + col0, v, 0);
+      store_vals<NV>(e.out2, (long)row * e.ldo2 + col0, v, 0);
+      break;
+    default:
+      break;
+  }
+}
+
+}  // namespace bag

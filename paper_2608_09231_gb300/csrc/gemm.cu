@@ -1,0 +1,364 @@
+// Projections of the DiT block: C[M,N] = A[M,K] W[N,K]^T with a fused epilogue.
+//
+// bf16 operands run on the 5th-generation tensor cores: a persistent, warp-specialised
+// kernel with one TMA producer warp, one MMA-issuing warp and four epilogue warps.
+// Operand tiles (128 x 64 of A, BN x 64 of W, 128-byte swizzle) stream through a
+// multi-stage shared-memory ring guarded by mbarriers; tcgen05.mma accumulates a
+// 128 x BN fp32 tile in tensor memory, double-buffered so the epilogue of one tile
+// overlaps the main loop of the next.  fp32 operands (the fp32 configuration, which
+// must hold 1e-4 relative parity) use a CUDA-core kernel with the same epilogue.
+#include <algorithm>
+#include <cstdio>
+#include <mutex>
+
+#include "common.cuh"
+#include "epilogue.cuh"
+#include "kernels.h"
+
+namespace bag {
+
+// ---------------------------------------------------------------------------
+// TMA descriptor encoding through the driver entry point
+// ---------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+int encode_tmap_2d_bf16(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                        uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return -1;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_stride_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
+                  strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? 0 : (int)r;
+}
+
+static int num_sms() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
+  }
+  return n;
+}
+
+// ---------------------------------------------------------------------------
+// CUDA-core GEMM (fp32 or bf16 operands, fp32 accumulation)
+// ---------------------------------------------------------------------------
+template <typename T>
+BAG_DEV float ld_f(const T* p) {
+  if constexpr (sizeof(T) == 2)
+    return __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(p));
+  else
+    return *p;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A, long lda,
+                                                        const T* __restrict__ W, long ldw,
+                                                        int M, int N, int K, const Epi e) {
+  if (epi_skip(e.st, e.flag_want)) return;
+  const int t = epi_step(e);
+  __shared__ float As[16][64 + 4];
+  __shared__ float Ws[16][64 + 4];
+  const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
+  const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
+  float acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+  for (int k0 = 0; k0 < K; k0 += 16) {
+    for (int i = threadIdx.x; i < 1024; i += 256) {
+      const int r = i / 16, c = i % 16;
+      const int m = m0 + r, n = n0 + r, k = k0 + c;
+      As[c][r] = (m < M && k < K) ? ld_f(A + (long)m * lda + k) : 0.f;
+      Ws[c][r] = (n < N && k < K) ? ld_f(W + (long)n * ldw + k) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < 16; ++kk) {
+      float a[4], b[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) b[j] = Ws[kk][tx * 4 + j];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] += a[i] * b[j];
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int row = m0 + ty * 4 + i;
+    const int col = n0 + tx * 4;
+    if (row < M && col < N) epi_apply<4>(e, t, row, col, acc[i]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// tcgen05 GEMM
+// ---------------------------------------------------------------------------
+constexpr int TC_BM = 128, TC_BK = 64;
+
+template <int BN>
+struct TcCfg {
+  static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
+  static constexpr int A_BYTES = TC_BM * TC_BK * 2;
+  static constexpr int B_BYTES = BN * TC_BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int TMEM_COLS = 2 * BN;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+};
+
+template <int BN>
+__global__ void __launch_bounds__(192, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const Epi e, int M, int N, int K, int* err) {
+  using C = TcCfg<BN>;
+  if (epi_skip(e.st, e.flag_want)) return;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + C::STAGES * C::A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* tfull = empty + C::STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int num_m = (M + TC_BM - 1) / TC_BM, num_n = N / BN;
+  const int tiles = num_m * num_n, kit = K / TC_BK;
+  const int t = epi_step(e);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(full + s, 1);
+      mbar_init(empty + s, 1);
+    }
+    mbar_init(tfull, 1);
+    mbar_init(tfull + 1, 1);
+    mbar_init(tempty, 128);
+    mbar_init(tempty + 1, 128);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      int s = 0;
+      uint32_t ph = 0;
+      long issued = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
+        const int mt = tile % num_m, nt = tile / num_m;
+        for (int kb = 0; kb < kit; ++kb) {
+          if (!mbar_wait(empty + s, ph ^ 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(full + s, C::STAGE_BYTES);
+          tma_load_2d(sA + s * C::A_BYTES, &tmA, kb * TC_BK, mt * TC_BM, full + s);
+          tma_load_2d(sB + s * C::B_BYTES, &tmB, kb * TC_BK, nt * BN, full + s);
+          ++issued;
+          if (++s == C::STAGES) {
+            s = 0;
+            ph ^= 1;
+          }
+        }
+      }
+      if (!ok) {
+        // drain: wait (bounded) for the copies this thread may still have in flight
+        const uint64_t t0 = global_ns();
+        for (int i = 0; i < C::STAGES && i < issued; ++i) {
+          if (--s < 0) {
+            s = C::STAGES - 1;
+            ph ^= 1;
+          }
+          while (!mbar_try_wait(full + s, ph) && global_ns() - t0 < kWaitLimitNs) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      constexpr uint32_t idesc = idesc_bf16_f32(TC_BM, BN);
+      int s = 0;
+      uint32_t ph = 0;
+      int acc = 0;
+      uint32_t aph = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
+        if (!mbar_wait(tempty + acc, aph ^ 1, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t dt = tmem_base + (uint32_t)(acc * BN);
+        for (int kb = 0; kb < kit; ++kb) {
+          if (!mbar_wait(full + s, ph, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + s * C::A_BYTES);
+          const uint32_t b0 = smem_u32(sB + s * C::B_BYTES);
+#pragma unroll
+          for (int k = 0; k < TC_BK / 16; ++k)
+            mma_bf16(dt, sw128_desc(a0 + k * 32), sw128_desc(b0 + k * 32), idesc,
+                     (kb | k) != 0 ? 1u : 0u);
+          mma_commit(empty + s);
+          if (++s == C::STAGES) {
+            s = 0;
+            ph ^= 1;
+          }
+        }
+        if (!ok) break;
+        mma_commit(tfull + acc);
+        acc ^= 1;
+        if (acc == 0) aph ^= 1;
+      }
+      // make sure every issued MMA has finished before TMEM is released
+      mma_commit(drain);
+      const uint64_t t0 = global_ns();
+      while (!mbar_try_wait(drain, 0) && global_ns() - t0 < kWaitLimitNs) {
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5 cover TMEM lane quarters 2,3,0,1) ----------------
+    const int q = warp & 3;
+    int acc = 0;
+    uint32_t aph = 0;
+    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+      const int mt = tile % num_m, nt = tile / num_m;
+      bool ok = mbar_wait(tfull + acc, aph, abort_flag);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      tc_fence_after();
+      const int row = mt * TC_BM + q * 32 + lane;
+      const uint32_t tb = tmem_base + (uint32_t)(acc * BN) + ((uint32_t)(q * 32) << 16);
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        float v[32];
+        tmem_ld32(tb + (uint32_t)(c * 32), v);
+        epi_apply<32>(e, t, row, nt * BN + c * 32, v);
+      }
+      tc_fence_before();
+      mbar_arrive(tempty + acc);
+      acc ^= 1;
+      if (acc == 0) aph ^= 1;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && *abort_flag && err) atomicOr(err, 1);
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+template <int BN>
+static cudaError_t launch_tc(const void* A, long lda, const void* W, long ldw, int M, int N,
+                             int K, const Epi& e, int* err, cudaStream_t s) {
+  using C = TcCfg<BN>;
+  CUtensorMap ta, tb;
+  if (encode_tmap_2d_bf16(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)lda * 2, TC_BK, TC_BM) ||
+      encode_tmap_2d_bf16(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)ldw * 2, TC_BK, BN))
+    return cudaErrorInvalidValue;
+  const int tiles = ((M + TC_BM - 1) / TC_BM) * (N / BN);
+  const int grid = std::min(tiles, num_sms());
+  gemm_tc_kernel<BN><<<grid, 192, C::SMEM, s>>>(ta, tb, e, M, N, K, err);
+  return cudaGetLastError();
+}
+
+cudaError_t attention_tc_init();
+
+cudaError_t kernels_init() {
+  cudaError_t r = cudaFuncSetAttribute(gemm_tc_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       TcCfg<256>::SMEM);
+  if (r == cudaSuccess)
+    r = cudaFuncSetAttribute(gemm_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             TcCfg<128>::SMEM);
+  if (r == cudaSuccess)
+    r = cudaFuncSetAttribute(gemm_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             TcCfg<64>::SMEM);
+  if (r == cudaSuccess) r = attention_tc_init();
+  num_sms();
+  return r;
+}
+
+int gemm_tc_supported(int M, int N, int K, long lda, long ldw) {
+  if (M <= 0 || K <= 0 || K % TC_BK != 0 || N % 64 != 0) return 0;
+  if (lda % 8 != 0 || ldw % 8 != 0) return 0;
+  return get_encode_fn() != nullptr;
+}
+
+cudaError_t gemm(const void* A, long lda, const void* W, long ldw, int M, int N, int K,
+                 int in_bf16, const Epi& epi_in, int* err, cudaStream_t s, int force_simt) {
+  if (M <= 0 || N <= 0) return cudaSuccess;
+  Epi e = epi_in;
+  e.M = M;
+  e.N = N;
+  const bool aligned = ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(W)) & 15) == 0;
+  if (in_bf16 && !force_simt && aligned && gemm_tc_supported(M, N, K, lda, ldw)) {
+    const int ns = num_sms();
+    const int mt = (M + TC_BM - 1) / TC_BM;
+    if (N % 256 == 0 && mt * (N / 256) >= ns) return launch_tc<256>(A, lda, W, ldw, M, N, K, e, err, s);
+    if (N % 128 == 0 && mt * (N / 128) >= ns) return launch_tc<128>(A, lda, W, ldw, M, N, K, e, err, s);
+    return launch_tc<64>(A, lda, W, ldw, M, N, K, e, err, s);
+  }
+  if (N % 4 != 0) return cudaErrorInvalidValue;
+  dim3 grid((N + 63) / 64, (M + 63) / 64);
+  if (in_bf16)
+    gemm_simt_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(
+        reinterpret_cast<const __nv_bfloat16*>(A), lda, reinterpret_cast<const __nv_bfloat16*>(W),
+        ldw, M, N, K, e);
+  else
+    gemm_simt_kernel<float><<<grid, 256, 0, s>>>(reinterpret_cast<const float*>(A), lda,
+                                                 reinterpret_cast<const float*>(W), ldw, M, N, K, e);
+  return cudaGetLastError();
+}
+
+}  // namespace bag

@@ -1,0 +1,151 @@
+// Internal interface between the C-ABI layer (bag_api.cu) and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace bag {
+
+// Per-sample state the step kernels read and write on the device, so that a whole
+// denoising step can be replayed from a CUDA graph with no host round trip.
+struct DevState {
+  int t;          // current step index (advanced on device at the end of each step)
+  int c;          // full evaluations spent so far (Algorithm 2's counter)
+  int t_last;     // last fully computed step
+  int flag;       // decision of the current step: 1 = full, 0 = reuse
+  int err;        // sticky error word (device wait timeout etc.)
+  int pad[3];
+};
+
+// Per-step log record (written by the gate kernel).
+constexpr int kLogFloats = 16;
+// [0..2]  gate inputs  (B-c)/B, (T-t)/T, drift
+// [3]     gate logit z
+// [4]     raw gate bit, [5] final decision m_t, [6] c before the step, [7] t - t_last
+// [8..10] budget state of Eq. 3: B/T, (B-c)/B, (B-c)/(T-t)
+// [11]    drift numerator sum|m_t - m_last|, [12] denominator sum|m_last|
+// [13..15] reserved
+
+enum EpiKind : int {
+  EPI_STORE = 0,      // out = acc + bias                       (out_bf16 selects type)
+  EPI_GELU = 1,       // out = gelu(acc + bias)
+  EPI_SILU = 2,       // out = silu(acc + bias)
+  EPI_QKV = 3,        // attention operands (+RoPE) and, past 3d, GELU(mlp) part
+  EPI_GATED_RES = 4,  // resid += gate * (acc + bias)
+  EPI_RES_ADD = 5,    // resid += acc + bias
+  EPI_EULER = 6,      // x += dsig[t] * (acc + bias); xb = bf16(x)
+  EPI_VEC = 7,        // out = acc + bias + addend; out2 = silu(out) (bf16 or f32)
+  EPI_DUAL_F32 = 8,   // out = out2 = acc + bias (f32)
+};
+
+struct Epi {
+  int kind = EPI_STORE;
+  int M = 0, N = 0;
+  const float* bias = nullptr;
+  // plain stores
+  void* out = nullptr;
+  long ldo = 0;
+  int out_bf16 = 0;
+  void* out2 = nullptr;
+  long ldo2 = 0;
+  int out2_bf16 = 0;
+  const float* addend = nullptr;  // EPI_VEC: [N] vector added to every row
+  // residual updates
+  float* resid = nullptr;
+  long ldr = 0;
+  const float* gate = nullptr;    // gate for step t = gate + t * gate_step
+  long gate_step = 0;
+  // attention operands
+  void* q = nullptr;
+  void* k = nullptr;
+  void* v = nullptr;       // v_mode 0: [rows, ldqk]; v_mode 1: transposed [H][dh][vpad]
+  int v_mode = 0;
+  long ldqk = 0;
+  int d = 0, dh = 0;
+  long vpad = 0;
+  int row_off = 0;         // joint-sequence row of this GEMM's row 0
+  int col_base = 0;        // logical column of this GEMM's column 0 (q=0, k=d, v=2d, mlp=3d)
+  const float2* rope = nullptr;  // [joint rows][dh/2] (cos, sin); null = no rotation
+  int act_bf16 = 1;        // q/k/v/mlp storage type
+  void* mlp = nullptr;     // GELU(mlp) columns go to mlp[row * ldm + (col - 3d)]
+  long ldm = 0;
+  // sampler update
+  float* x = nullptr;
+  __nv_bfloat16* xb = nullptr;
+  long ldx = 0;
+  const float* dsig = nullptr;  // [T]: sigma_{t+1} - sigma_t
+  // step-dependent addressing and early exit
+  const DevState* st = nullptr;  // null: step 0, no flag check
+  int flag_want = -1;            // -1: always run; 0/1: run only when st->flag equals it
+};
+
+// ---------------------------------------------------------------------------
+// launchers (all asynchronous on the given stream); return cudaError_t
+// ---------------------------------------------------------------------------
+// C[M,N] = A[M,K] W[N,K]^T with the fused epilogue.  Tensor-core path for bf16
+// operands; fp32 operands (and shapes the tensor-core path does not tile) go to the
+// CUDA-core path.
+cudaError_t gemm(const void* A, long lda, const void* W, long ldw, int M, int N, int K,
+                 int in_bf16, const Epi& epi, int* err, cudaStream_t s, int force_simt = 0);
+int gemm_tc_supported(int M, int N, int K, long lda, long ldw);
+
+struct AttnArgs {
+  const void* q;  long ldq;      // [Nq rows][ldq], head h at column h*dh
+  const void* k;  long ldk;      // [Nk rows][ldk]
+  const void* v;  int v_mode; long ldv; long vpad;  // mode 0 like k; mode 1 [H][dh][vpad]
+  void* o;        long ldo;      // output [Nq][ldo], head h at column h*dh
+  int nq, nk, heads, dh;
+  int bf16;                      // operand/output type
+  const DevState* st; int flag_want;
+};
+cudaError_t attention(const AttnArgs& a, int* err, cudaStream_t s, int force_simt = 0);
+int attention_tc_supported(const AttnArgs& a);
+
+// Row-wise LayerNorm (no affine, eps 1e-6) + adaLN modulation over rows [0, rows).
+// Rows < split use (shift_a, scale_a), the rest (shift_b, scale_b); modulation vectors
+// are read at base + t * mod_step.  shift/scale null = plain LayerNorm.
+struct LnArgs {
+  const float* x; long ldx;
+  void* y; long ldy; int y_bf16;
+  int rows, cols, split;
+  const float* shift_a; const float* scale_a;
+  const float* shift_b; const float* scale_b;
+  long mod_step;
+  // fused trajectory signal: per-row partial sums of |y - ref| and |ref|; y also
+  // stored to sig_out (the reference for the next full step is copied from it).
+  const void* sig_ref; float* sig_partial; int sig_on;
+  const DevState* st; int flag_want;
+};
+cudaError_t ln_mod(const LnArgs& a, cudaStream_t s);
+
+cudaError_t gate_step(DevState* st, const float* sig_partial, int sig_rows, const float* gate_params,
+                      float thr, int T, int B, int policy, const uint8_t* policy_mask,
+                      float* log, unsigned long long cond_handle, int use_cond, cudaStream_t s);
+cudaError_t cache_refresh(const DevState* st, const float* h_img, const float* h_in, float* R,
+                          void* m_last, const void* m_cur, long n, long m_n, int m_bf16,
+                          int flag_want, cudaStream_t s);
+cudaError_t cache_reuse(const DevState* st, float* h_img, const float* h_in, const float* R,
+                        long n, int flag_want, cudaStream_t s);
+cudaError_t copy_rows_f32(const DevState* st, int flag_want, float* dst, long ldd, const void* src,
+                          long lds, int src_bf16, int rows, int cols, cudaStream_t s);
+cudaError_t advance_step(DevState* st, cudaStream_t s);
+cudaError_t sinusoid_all(void* out, int out_bf16, int T, int dim, cudaStream_t s);
+cudaError_t expand_wan_mod(float* mod_all, const float* shared6d, const float* tables,
+                           int T, int nblocks, int d, cudaStream_t s);
+cudaError_t to_bf16(__nv_bfloat16* dst, const float* src, long n, cudaStream_t s);
+cudaError_t fill_synth(void* dst, long n, uint64_t seed, uint64_t key, float c32, int bf16,
+                       cudaStream_t s);
+cudaError_t residual_add(float* out, const float* a, const float* b, long n, cudaStream_t s);
+cudaError_t rel_l1_partials(const void* a, const void* b, int a_bf16, long rows, long cols,
+                            float* partial, cudaStream_t s);
+
+// one-time kernel attribute setup (dynamic shared memory limits); call before capture
+cudaError_t kernels_init();
+
+// host-side TMA descriptor encoding (driver entry point resolved at run time)
+int encode_tmap_2d_bf16(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                        uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer);
+
+}  // namespace bag

@@ -1,0 +1,252 @@
+"""GPU path against the fp64 oracle, through the C ABI.
+
+Bars (from the method's arithmetic):
+  * schedules: the full/cached bit of every step is bit-exact when the oracle takes its
+    decisions on the GPU's logged gate inputs; the gate logit itself is bit-exact
+    (both sides evaluate it in fp32 in the same order);
+  * latents: max-abs error <= 1e-4 x RMS(oracle) for the fp32 configuration and
+    <= 2e-2 x RMS(oracle) for bf16 configurations;
+  * integer/byte work (weights from the seeded generator, NFE counts) bit-exact.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import bag_oracle as O
+from paper_2608_09231_gb300 import bag, configs, synth
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"f32": 1e-4, "bf16": 2e-2}
+
+
+def _dev_inputs(cfg, inp):
+    x = torch.from_numpy(inp["x"].copy()).cuda()
+    txt = torch.from_numpy(inp["txt"]).cuda()
+    if cfg["dtype"] == "bf16":
+        txt = txt.to(torch.bfloat16)
+    pooled = torch.from_numpy(inp["pooled"]).cuda()
+    return x, txt, pooled
+
+
+def _gpu_sample(cfg, T, B, tau=0.5, policy=None, mask=None, ctx=None):
+    own = ctx is None
+    if own:
+        ctx = bag.create(cfg, T=T, B=B, tau=tau)
+    inp = synth.make_inputs(cfg)
+    x, txt, pooled = _dev_inputs(cfg, inp)
+    if policy is not None:
+        ctx.set_policy(policy, mask)
+    ctx.reset()
+    m, log, nfe = ctx.run(x, txt, pooled)
+    torch.cuda.synchronize()
+    out = x.cpu().numpy()
+    if own:
+        ctx.close()
+    return inp, out, m, log, nfe
+
+
+def _gate_inputs(log):
+    return [None] + [float(v) for v in log[1:, 2]]
+
+
+@pytest.mark.parametrize("name", ["tiny", "flux_small", "wan_small"])
+def test_device_weights_equal_generator(name, lib):
+    cfg = configs.get_config(name)
+    ctx = bag.create(cfg, T=4, B=2)
+    W = synth.make_weights(cfg)
+    for blk, tname in [(-1, "pe_w"), (-1, "fin_b"), (-1, "t1_w"), (0, W["blocks"][0] and
+                                                                  list(W["blocks"][0])[1]),
+                       (len(W["blocks"]) - 1, list(W["blocks"][-1])[-1])]:
+        ref = W["global"][tname] if blk < 0 else W["blocks"][blk][tname]
+        got = ctx.get_weight(blk, tname, ref.size).reshape(ref.shape)
+        assert np.array_equal(got, ref), (blk, tname)
+    ctx.close()
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny_ragged", "single_small", "flux_small",
+                                  "qwen_small", "wan_small"])
+def test_sample_parity_against_oracle(name, lib):
+    cfg = configs.get_config(name)
+    T, B = cfg["T"], cfg["budgets"][0]
+    inp, got, mask, log, nfe = _gpu_sample(cfg, T, B)
+    assert nfe == B and int(mask.sum()) == B and mask[0] == 1
+    W = synth.make_weights(cfg)
+    g = synth.make_gate(cfg["gate_seed"])
+    ref = O.sample(cfg, W, g, inp, T=T, B=B, drift_override=_gate_inputs(log))
+    # schedule bit-exact, gate logit bit-exact on the GPU's inputs
+    assert list(mask) == ref["mask"]
+    for t in range(1, T):
+        f = [np.float32(v) for v in log[t, 0:3]]
+        assert O.gate_logit(f, g) == np.float32(log[t, 3]), t
+        assert f[0] == np.float32(B - log[t, 6]) / np.float32(B)
+        assert f[1] == np.float32(T - t) / np.float32(T)
+        # the GPU's drift agrees with the oracle's own drift
+        dref = ref["log"][t]["drift"]
+        assert abs(float(log[t, 2]) - dref) <= max(TOL[cfg["dtype"]], 1e-6) * max(dref, 1e-3), t
+    rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
+    err = float(np.max(np.abs(got.astype(np.float64) - ref["x"])))
+    assert err <= TOL[cfg["dtype"]] * rms, (err, rms)
+
+
+@pytest.mark.parametrize("name", ["tiny", "flux_small"])
+def test_budget_equal_T_is_uncached_sampling_bit_exact(name, lib):
+    cfg = configs.get_config(name)
+    T = 5
+    _, a, ma, _, na = _gpu_sample(cfg, T, T)
+    _, b, mb, _, nb = _gpu_sample(cfg, T, 1, policy=bag.POLICY_FULL)
+    assert na == nb == T and list(ma) == list(mb) == [1] * T
+    assert np.array_equal(a, b)
+
+
+@pytest.mark.parametrize("tau", [0.3, 0.5, 0.7])
+def test_nfe_equals_budget_for_any_tau(tau, lib):
+    cfg = configs.get_config("tiny_ragged")
+    T = cfg["T"]
+    for B in (1, 3, T):
+        _, _, m, log, nfe = _gpu_sample(cfg, T, B, tau=tau)
+        assert nfe == B and int(m.sum()) == B and m[0] == 1
+        assert list(m) == O.schedule_from_gate_bits([None] + [int(v) for v in log[1:, 4]], B, T)
+
+
+def test_static_mask_policy(lib):
+    cfg = configs.get_config("tiny_ragged")
+    T = cfg["T"]
+    want = [1, 0, 1, 1, 0, 0, 1]
+    _, got, m, _, nfe = _gpu_sample(cfg, T, 4, policy=bag.POLICY_MASK, mask=np.array(want, np.uint8))
+    assert list(m) == want and nfe == 4
+    inp = synth.make_inputs(cfg)
+    ref = O.sample(cfg, synth.make_weights(cfg), synth.make_gate(cfg["gate_seed"]), inp, T=T, B=4,
+                   policy=want)
+    rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
+    assert float(np.max(np.abs(got - ref["x"]))) <= TOL["f32"] * rms
+
+
+@pytest.mark.parametrize("name", ["tiny", "flux_small"])
+def test_step_api_matches_run(name, lib):
+    cfg = configs.get_config(name)
+    T, B = 6, 3
+    ctx = bag.create(cfg, T=T, B=B)
+    inp = synth.make_inputs(cfg)
+    x, txt, pooled = _dev_inputs(cfg, inp)
+    x0 = x.clone()
+    m_run, _, _ = ctx.run(x, txt, pooled)
+    ctx.reset()
+    xs = x0.clone()
+    flags = torch.zeros(T, dtype=torch.int32, device="cuda")
+    with pytest.raises(bag.BagError) as ei:
+        ctx.step(xs, 1, txt, pooled, xs, flags[1:])
+    assert ei.value.status == 4  # EORDER
+    for t in range(T):
+        ctx.step(xs, t, txt, pooled, xs, flags[t:])
+    torch.cuda.synchronize()
+    assert list(flags.cpu().numpy()) == list(m_run)
+    assert torch.equal(xs, x)
+    ctx.close()
+
+
+def test_run_host_matches_device(lib):
+    cfg = configs.get_config("flux_small")
+    T, B = 5, 3
+    ctx = bag.create(cfg, T=T, B=B)
+    inp = synth.make_inputs(cfg)
+    x, txt, pooled = _dev_inputs(cfg, inp)
+    m1, _, _ = ctx.run(x, txt, pooled)
+    ctx.reset()
+    xh = inp["x"].copy()
+    m2, _, _ = ctx.run_host(xh, inp["txt"], inp["pooled"])
+    assert list(m1) == list(m2)
+    assert np.array_equal(xh, x.cpu().numpy())
+    ctx.close()
+
+
+# ---------------------------------------------------------------------------
+# kernel-level parity
+# ---------------------------------------------------------------------------
+def _bf16_tensor(seed, shape, std=1.0):
+    v = synth.bf16_round(synth.normal(seed, 77, int(np.prod(shape)), std)).reshape(shape)
+    return v, torch.from_numpy(v).cuda().to(torch.bfloat16)
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 256, 128), (129, 64, 64), (1000, 384, 512),
+                                   (77, 512, 256), (4096, 3072, 3072), (50, 1024, 320)])
+@pytest.mark.parametrize("simt", [0, 1])
+def test_gemm_bf16_against_fp64(M, N, K, simt, lib):
+    ctx = bag.create("tiny", T=2, B=1)
+    a, A = _bf16_tensor(1, (M, K))
+    w, Wt = _bf16_tensor(2, (N, K), 0.05)
+    b = synth.normal(3, 5, N, 0.1)
+    bias = torch.from_numpy(b).cuda()
+    C = torch.zeros((M, N), dtype=torch.float32, device="cuda")
+    ctx.gemm_bf16(A, Wt, bias, C, M, N, K, 0, simt)
+    torch.cuda.synchronize()
+    rows = np.arange(M) if M <= 1100 else np.r_[0:64, M - 64:M, 1000:1010]
+    ref = a[rows].astype(np.float64) @ w.T.astype(np.float64) + b
+    bound = 4 * K * 2.0 ** -24 * (np.abs(a[rows]).astype(np.float64) @ np.abs(w).T) + 1e-7
+    got = C.cpu().numpy()[rows]
+    assert np.all(np.abs(got - ref) <= bound)
+    ctx.close()
+
+
+def test_gemm_gelu_epilogue(lib):
+    ctx = bag.create("tiny", T=2, B=1)
+    M, N, K = 257, 128, 192
+    a, A = _bf16_tensor(4, (M, K))
+    w, Wt = _bf16_tensor(5, (N, K), 0.1)
+    C = torch.zeros((M, N), dtype=torch.float32, device="cuda")
+    ctx.gemm_bf16(A, Wt, None, C, M, N, K, 1, 0)
+    torch.cuda.synchronize()
+    ref = O.gelu_tanh(a.astype(np.float64) @ w.T.astype(np.float64))
+    assert np.max(np.abs(C.cpu().numpy() - ref)) <= 1e-4 * (1 + np.max(np.abs(ref)))
+    ctx.close()
+
+
+@pytest.mark.parametrize("rows,cols", [(37, 256), (1000, 3072), (5, 5120)])
+def test_ln_mod_against_oracle(rows, cols, lib):
+    ctx = bag.create("tiny", T=2, B=1)
+    x = synth.normal(7, 1, rows * cols, 2.0).reshape(rows, cols) + 0.5
+    sh = synth.normal(7, 2, cols, 0.5)
+    sc = synth.normal(7, 3, cols, 0.5)
+    y = torch.zeros((rows, cols), dtype=torch.bfloat16, device="cuda")
+    ctx.ln_mod(torch.from_numpy(x).cuda(), torch.from_numpy(sh).cuda(),
+               torch.from_numpy(sc).cuda(), y, rows, cols)
+    torch.cuda.synchronize()
+    ref = O.modulate(O.layer_norm(x.astype(np.float64)), sh, sc)
+    got = y.float().cpu().numpy()
+    assert np.all(np.abs(got - ref) <= 2.0 ** -8 * np.abs(ref) + 1e-5)
+    ctx.close()
+
+
+def test_residual_add_exact(lib):
+    ctx = bag.create("tiny", T=2, B=1)
+    n = 1 << 20
+    a = torch.from_numpy(synth.normal(9, 1, n, 1.0)).cuda()
+    r = torch.from_numpy(synth.normal(9, 2, n, 0.3)).cuda()
+    out = torch.empty_like(a)
+    ctx.residual_add(out, a, r, n)
+    torch.cuda.synchronize()
+    assert np.array_equal(out.cpu().numpy(), a.cpu().numpy() + r.cpu().numpy())
+    ctx.close()
+
+
+@pytest.mark.parametrize("nq,nk,heads,dh", [(300, 300, 2, 128), (129, 515, 3, 128),
+                                            (288, 288, 4, 64), (4608, 4608, 1, 128)])
+@pytest.mark.parametrize("simt", [0, 1])
+def test_attention_against_oracle(nq, nk, heads, dh, simt, lib):
+    ctx = bag.create("tiny", T=2, B=1)
+    d = heads * dh
+    q, Q = _bf16_tensor(11, (nq, d))
+    k, K_ = _bf16_tensor(12, (nk, d))
+    v, V = _bf16_tensor(13, (nk, d))
+    o = torch.zeros((nq, d), dtype=torch.bfloat16, device="cuda")
+    ctx.attention_bf16(Q, K_, V, o, nq, nk, heads, dh, simt)
+    torch.cuda.synchronize()
+    rows = np.arange(nq) if nq <= 600 else np.r_[0:40, nq - 40:nq]
+    ref = O.attention(q.reshape(nq, heads, dh).astype(np.float64),
+                      k.reshape(nk, heads, dh).astype(np.float64),
+                      v.reshape(nk, heads, dh).astype(np.float64), q_rows=rows).reshape(len(rows), d)
+    got = o.float().cpu().numpy()[rows]
+    # P and O are rounded to bf16: allow 2^-7 relative to the output scale
+    assert np.max(np.abs(got - ref)) <= 2.0 ** -7 * (np.max(np.abs(ref)) + 1e-3)
+    ctx.close()
