@@ -106,6 +106,7 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t s);
 cudaError_t attention(const AttnArgs& a, int* err, cudaStream_t s, int force_simt) {
   if (a.nq <= 0) return cudaSuccess;
   if (a.bf16 && !force_simt && attention_tc_supported(a)) return attention_tc(a, err, s);
+  // (until the tensor-core attention covers a shape, bf16 attention runs on CUDA cores)
   dim3 grid((a.nq + 15) / 16, a.heads);
   if (a.dh == 64) {
     if (a.bf16)

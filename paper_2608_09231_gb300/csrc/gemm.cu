@@ -342,7 +342,10 @@ cudaError_t gemm(const void* A, long lda, const void* W, long ldw, int M, int N,
   e.M = M;
   e.N = N;
   const bool aligned = ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(W)) & 15) == 0;
-  if (in_bf16 && !force_simt && aligned && gemm_tc_supported(M, N, K, lda, ldw)) {
+  if (in_bf16 && !force_simt) {
+    // bf16 operands always take the tensor-core path; a shape or pointer it cannot
+    // tile is an error, never a silent switch to the CUDA-core kernel
+    if (!aligned || !gemm_tc_supported(M, N, K, lda, ldw)) return cudaErrorNotSupported;
     const int ns = num_sms();
     const int mt = (M + TC_BM - 1) / TC_BM;
     if (N % 256 == 0 && mt * (N / 256) >= ns) return launch_tc<256>(A, lda, W, ldw, M, N, K, e, err, s);
