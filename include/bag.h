@@ -108,8 +108,9 @@ void bag_destroy(bag_ctx* ctx);
  * null).  Valid until the next call on the context. */
 const char* bag_last_error(bag_ctx* ctx);
 
-/* Make later work run on `cuda_stream` (a cudaStream_t; null = the legacy stream).
- * Invalidates captured step graphs (they are re-captured on first use). */
+/* Order the context's work after, and before, the caller's `cuda_stream` (a
+ * cudaStream_t; null = the legacy stream).  The context keeps its own stream for the
+ * captured step graph and bridges the two with events on every call. */
 bag_status bag_set_stream(bag_ctx* ctx, void* cuda_stream);
 
 /* Replace the gate parameters (Eq. 1; App. A.2 z-scored inputs).  theta: host array of
@@ -164,6 +165,30 @@ bag_status bag_forward_block(bag_ctx* ctx, int block, int t_mod, float* h);
  * modulation for all T steps) and stage its text tokens; bag_run does this itself. */
 bag_status bag_prepare(bag_ctx* ctx, const bag_cond* cond);
 
+/* Profiled sample.  Same as bag_run on a fresh sample, but every kernel is launched
+ * directly (no graph) between two CUDA events, and the step's decision is read back
+ * after the gate so that only the taken branch is launched.  out[BAG_PROF_KINDS]
+ * receives per kernel class: launches, summed event time (ms), summed algorithmic
+ * flops and bytes (the work the method needs, not counter values).  Slower than
+ * bag_run (one host synchronisation per step); for measurement only. */
+enum {
+  BAG_PROF_GEMM = 0,   /* projections (tensor cores), incl. patch embed and final layer */
+  BAG_PROF_ATTN = 1,   /* attention */
+  BAG_PROF_NORM = 2,   /* LayerNorm + modulation inside the stack and the final layer */
+  BAG_PROF_SIGNAL = 3, /* trajectory signal (block-0 LN-mod fused with the rel-L1 partials) */
+  BAG_PROF_GATE = 4,   /* gate + pacing */
+  BAG_PROF_CACHE = 5,  /* cache refresh (full step) and residual reuse (cached step) */
+  BAG_PROF_KINDS = 6
+};
+typedef struct {
+  long launches;
+  double ms;
+  double flops;
+  double bytes;
+} bag_prof_entry;
+bag_status bag_profile_run(bag_ctx* ctx, float* x_inout, const bag_cond* cond, bag_stats* stats,
+                           bag_prof_entry* out);
+
 /* Number of kernel launches the last bag_run enqueued (graph nodes included). */
 bag_status bag_launch_count(bag_ctx* ctx, long* out);
 
@@ -175,10 +200,14 @@ bag_status bag_gemm_bf16(bag_ctx* ctx, const void* A, long lda, const void* W, l
                          const float* bias, float* C, long ldc, int M, int N, int K,
                          int epilogue, int force_simt);
 
-/* Multi-head attention softmax(q k^T / sqrt(dh)) v: q [nq, ld], k, v [nk, ld] bf16 device,
- * head h at columns [h*dh, (h+1)*dh); o [nq, ld] bf16 device.  dh = 64 or 128. */
+/* Multi-head attention softmax(q k^T / sqrt(dh)) v (the joint attention of the DiT
+ * blocks): q [nq, ld], k [nk, ld] bf16 device, head h at columns [h*dh, (h+1)*dh);
+ * o [nq, ld] bf16 device.  v: if vpad > 0, transposed per head, [heads][dh][vpad] bf16
+ * (vpad >= nk, multiple of 8; the layout the tensor-core kernel reads); if vpad == 0,
+ * [nk, ld] like k (CUDA-core kernel only).  The tensor-core kernel needs dh = 128;
+ * force_simt != 0 selects the CUDA-core kernel (dh 64 or 128). */
 bag_status bag_attention_bf16(bag_ctx* ctx, const void* q, const void* k, const void* v,
-                              void* o, long ld, int nq, int nk, int heads, int dh,
+                              void* o, long ld, int nq, int nk, int heads, int dh, long vpad,
                               int force_simt);
 
 /* y = (1 + scale) * LayerNorm(x) + shift row-wise (eps 1e-6, no affine): x fp32 device

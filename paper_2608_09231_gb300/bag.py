@@ -26,7 +26,10 @@ STATUS = {0: "BAG_OK", 1: "BAG_EINVAL", 2: "BAG_ENOMEM", 3: "BAG_ECUDA", 4: "BAG
 EXPORTS = ["bag_create", "bag_destroy", "bag_last_error", "bag_set_stream", "bag_load_gate",
            "bag_set_policy", "bag_reset", "bag_step", "bag_run", "bag_run_host",
            "bag_get_weight", "bag_forward_block", "bag_prepare", "bag_launch_count",
-           "bag_gemm_bf16", "bag_attention_bf16", "bag_ln_mod", "bag_residual_add"]
+           "bag_gemm_bf16", "bag_attention_bf16", "bag_ln_mod", "bag_residual_add",
+           "bag_profile_run"]
+
+PROF_KINDS = ["gemm", "attention", "norm", "signal", "gate", "cache"]
 
 
 class BagError(RuntimeError):
@@ -46,6 +49,11 @@ class Arch(ctypes.Structure):
 
 class Cond(ctypes.Structure):
     _fields_ = [("txt", ctypes.c_void_p), ("pooled", ctypes.c_void_p)]
+
+
+class ProfEntry(ctypes.Structure):
+    _fields_ = [("launches", ctypes.c_long), ("ms", ctypes.c_double), ("flops", ctypes.c_double),
+                ("bytes", ctypes.c_double)]
 
 
 class Stats(ctypes.Structure):
@@ -85,9 +93,11 @@ def load(path=None):
         "bag_prepare": ([_P, ctypes.POINTER(Cond)], _I),
         "bag_launch_count": ([_P, ctypes.POINTER(_L)], _I),
         "bag_gemm_bf16": ([_P, _P, _L, _P, _L, _P, _P, _L, _I, _I, _I, _I, _I], _I),
-        "bag_attention_bf16": ([_P, _P, _P, _P, _P, _L, _I, _I, _I, _I, _I], _I),
+        "bag_attention_bf16": ([_P, _P, _P, _P, _P, _L, _I, _I, _I, _I, _L, _I], _I),
         "bag_ln_mod": ([_P, _P, _P, _P, _P, _I, _I], _I),
         "bag_residual_add": ([_P, _P, _P, _P, _L], _I),
+        "bag_profile_run": ([_P, _P, ctypes.POINTER(Cond), ctypes.POINTER(Stats),
+                             ctypes.POINTER(ProfEntry)], _I),
     }
     for name, (args, res) in sig.items():
         f = getattr(lib, name)
@@ -186,6 +196,17 @@ class Context:
         self._chk(self.lib.bag_run(self.h, _ptr(x), ctypes.byref(c), ctypes.byref(s)))
         return mask, log, s.nfe
 
+    def profile_run(self, x, txt, pooled):
+        """Profiled sample (direct launches with events); returns (mask, log, nfe, prof)
+        where prof maps a kernel class to dict(launches, ms, flops, bytes)."""
+        c = Cond(txt.data_ptr(), None if pooled is None else pooled.data_ptr())
+        s, mask, log = self._stats()
+        out = (ProfEntry * len(PROF_KINDS))()
+        self._chk(self.lib.bag_profile_run(self.h, _ptr(x), ctypes.byref(c), ctypes.byref(s), out))
+        prof = {k: dict(launches=out[i].launches, ms=out[i].ms, flops=out[i].flops,
+                        bytes=out[i].bytes) for i, k in enumerate(PROF_KINDS)}
+        return mask, log, s.nfe, prof
+
     def run_host(self, x, txt, pooled):
         """All T steps with host numpy buffers (x updated in place); returns (mask, log, nfe)."""
         assert x.dtype == np.float32 and x.flags.c_contiguous
@@ -217,9 +238,10 @@ class Context:
                                          _ptr(bias), _ptr(C), C.stride(0), M, N, K, epilogue,
                                          force_simt))
 
-    def attention_bf16(self, q, k, v, o, nq, nk, heads, dh, force_simt=0):
+    def attention_bf16(self, q, k, v, o, nq, nk, heads, dh, vpad=0, force_simt=0):
+        """v: [nk, ld] when vpad == 0, else transposed per head [heads, dh, vpad]."""
         self._chk(self.lib.bag_attention_bf16(self.h, _ptr(q), _ptr(k), _ptr(v), _ptr(o),
-                                              q.stride(0), nq, nk, heads, dh, force_simt))
+                                              q.stride(0), nq, nk, heads, dh, vpad, force_simt))
 
     def ln_mod(self, x, shift, scale, y, rows, cols):
         self._chk(self.lib.bag_ln_mod(self.h, _ptr(x), _ptr(shift), _ptr(scale), _ptr(y), rows,

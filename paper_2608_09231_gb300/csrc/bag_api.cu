@@ -146,6 +146,17 @@ struct bag_ctx {
 
   int next_t = 0;
   bool prepared = false;
+
+  // per-launch profiling (direct launches only)
+  struct ProfRec {
+    int kind;
+    double flops, bytes;
+    int e0, e1;
+  };
+  std::vector<ProfRec> prof;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_used = 0;
+  bool profiling = false;
 };
 
 static std::string g_create_error;
@@ -504,14 +515,43 @@ static bag_status alloc_activations(bag_ctx* ctx) {
 // ---------------------------------------------------------------------------
 // enqueue helpers
 // ---------------------------------------------------------------------------
+static int prof_event(bag_ctx* ctx) {
+  if (ctx->ev_used == ctx->ev_pool.size()) {
+    cudaEvent_t ev;
+    if (cudaEventCreate(&ev) != cudaSuccess) return -1;
+    ctx->ev_pool.push_back(ev);
+  }
+  return (int)ctx->ev_used++;
+}
+
 struct Enq {
   bag_ctx* ctx;
   cudaStream_t s;
   long* count;
   cudaError_t e = cudaSuccess;
+  int pk = -1, pe0 = -1;
+  double pf = 0, pb = 0;
+  // announce the next launch (kind, algorithmic flops and bytes) for profiling
+  void pre(int kind, double flops, double bytes) {
+    if (!ctx->profiling) return;
+    pe0 = prof_event(ctx);
+    if (pe0 < 0) return;
+    cudaEventRecord(ctx->ev_pool[pe0], s);
+    pk = kind;
+    pf = flops;
+    pb = bytes;
+  }
   void chk(cudaError_t r) {
     if (e == cudaSuccess && r != cudaSuccess) e = r;
     if (count) ++*count;
+    if (pk >= 0) {
+      const int pe1 = prof_event(ctx);
+      if (pe1 >= 0) {
+        cudaEventRecord(ctx->ev_pool[pe1], s);
+        ctx->prof.push_back({pk, pf, pb, pe0, pe1});
+      }
+      pk = -1;
+    }
   }
 };
 
@@ -529,6 +569,13 @@ static inline void* off_act(const bag_ctx* ctx, void* p, long elems) {
 
 static void enq_gemm(Enq& q, const void* A, long lda, const Tensor& W, long ldw, int M, int N,
                      int K, const Epi& e) {
+  {
+    const double es = (double)q.ctx->act_size;
+    double out = (double)M * N * 4;
+    if (e.kind == EPI_GATED_RES || e.kind == EPI_RES_ADD) out = (double)M * N * 8;
+    else if (e.kind == EPI_QKV || e.kind == EPI_GELU) out = (double)M * N * es;
+    q.pre(BAG_PROF_GEMM, 2.0 * M * N * K, ((double)M + N) * K * es + out);
+  }
   q.chk(gemm(A, lda, W.p, ldw, M, N, K, q.ctx->act_bf16, e, q.ctx->st ? &q.ctx->st->err : nullptr, q.s));
 }
 
@@ -551,6 +598,7 @@ static void enq_ln(Enq& q, const float* x, long ldx, void* y, long ldy, int rows
   a.mod_step = q.ctx->mod_stride;
   a.st = st;
   a.flag_want = flag_want;
+  q.pre(BAG_PROF_NORM, 0.0, (double)rows * q.ctx->d * (4.0 + q.ctx->act_size));
   q.chk(ln_mod(a, q.s));
 }
 
@@ -592,6 +640,8 @@ static void enq_attn(Enq& q, const void* Q, const void* K, const void* V, long v
   a.bf16 = ctx->act_bf16;
   a.st = st;
   a.flag_want = flag_want;
+  q.pre(BAG_PROF_ATTN, 4.0 * nq * nk * ctx->H * ctx->dh,
+        ((double)nq * 2 + 2.0 * nk) * ctx->d * ctx->act_size);
   q.chk(attention(a, ctx->st ? &ctx->st->err : nullptr, q.s));
 }
 
@@ -792,7 +842,9 @@ static void enq_prefix(Enq& q, int use_cond, unsigned long long handle) {
   a.sig_on = 1;
   a.st = ctx->st;
   a.flag_want = -1;
+  q.pre(BAG_PROF_SIGNAL, 0.0, (double)ctx->ni * d * (4.0 + 2.0 * ctx->act_size));
   q.chk(ln_mod(a, q.s));
+  q.pre(BAG_PROF_GATE, 0.0, (double)ctx->ni * 8);
   q.chk(gate_step(ctx->st, ctx->sig_partial, ctx->ni, ctx->d_gate, ctx->thr, ctx->T, ctx->B,
                   ctx->policy, ctx->d_pmask, ctx->log, handle, use_cond, q.s));
 }
@@ -803,12 +855,14 @@ static void enq_full(Enq& q, int fw) {
   if (ctx->arch.kind != BAG_KIND_WAN)
     q.chk(copy_rows_f32(ctx->st, fw, ctx->hj, d, ctx->txt_stage, d, ctx->act_bf16, ctx->nx, (int)d, q.s));
   for (int b = 0; b < ctx->nblk; ++b) enq_block(q, b, ctx->hj, ctx->st, fw);
+  q.pre(BAG_PROF_CACHE, 0.0, (double)ctx->ni * d * (12.0 + 2.0 * ctx->act_size));
   q.chk(cache_refresh(ctx->st, img_stream(ctx), ctx->h_in, ctx->R, ctx->m_last, ctx->m_cur,
                       (long)ctx->ni * d, (long)ctx->ni * d, ctx->act_bf16, fw, q.s));
 }
 
 static void enq_skip(Enq& q, int fw) {
   bag_ctx* ctx = q.ctx;
+  q.pre(BAG_PROF_CACHE, 0.0, (double)ctx->ni * ctx->d * 12.0);
   q.chk(cache_reuse(ctx->st, img_stream(ctx), ctx->h_in, ctx->R, (long)ctx->ni * ctx->d, fw, q.s));
 }
 
@@ -974,6 +1028,67 @@ static bag_status launch_step(bag_ctx* ctx) {
   return BAG_OK;
 }
 
+// Profiled sample: direct launches, each bracketed by events; the decision is read back
+// after every gate so that only the taken branch is launched (and timed).
+static bag_status profile_run_impl(bag_ctx* ctx, float* x_inout, const bag_cond* cond,
+                                   bag_stats* stats, bag_prof_entry* out) {
+  if (!x_inout || !out) return fail(ctx, BAG_EINVAL, "null argument");
+  if (ctx->next_t != 0) return fail(ctx, BAG_ESTATE, "needs a fresh sample (bag_reset)");
+  ctx->prof.clear();
+  ctx->ev_used = 0;
+  ctx->profiling = true;
+  bag_status s = enq_prepare(ctx, cond);
+  const size_t xbytes = (size_t)ctx->ni * ctx->C * 4;
+  int nfe = 0;
+  std::vector<float> lg((size_t)ctx->T * kLogFloats);
+  if (s == BAG_OK) {
+    cudaMemcpyAsync(ctx->x, x_inout, xbytes, cudaMemcpyDeviceToDevice, ctx->stream);
+    if (ctx->act_bf16) to_bf16(ctx->xb, ctx->x, (long)ctx->ni * ctx->C, ctx->stream);
+    for (int t = 0; t < ctx->T && s == BAG_OK; ++t) {
+      long cnt = 0;
+      Enq q{ctx, ctx->stream, &cnt};
+      enq_prefix(q, 0, 0);
+      int flag = 0;
+      if (cudaMemcpyAsync(&flag, &ctx->st->flag, 4, cudaMemcpyDeviceToHost, ctx->stream) != cudaSuccess ||
+          cudaStreamSynchronize(ctx->stream) != cudaSuccess) {
+        s = fail(ctx, BAG_ECUDA, "profile sync failed");
+        break;
+      }
+      nfe += flag;
+      if (flag)
+        enq_full(q, 1);
+      else
+        enq_skip(q, 0);
+      enq_suffix(q);
+      if (q.e != cudaSuccess) s = fail(ctx, BAG_ECUDA, std::string("profile step: ") + cudaGetErrorString(q.e));
+    }
+    cudaMemcpyAsync(x_inout, ctx->x, xbytes, cudaMemcpyDeviceToDevice, ctx->stream);
+    cudaMemcpyAsync(lg.data(), ctx->log, lg.size() * 4, cudaMemcpyDeviceToHost, ctx->stream);
+    if (cudaStreamSynchronize(ctx->stream) != cudaSuccess && s == BAG_OK) s = fail(ctx, BAG_ECUDA, "profile sync");
+  }
+  ctx->profiling = false;
+  ctx->next_t = ctx->T;
+  for (int k = 0; k < BAG_PROF_KINDS; ++k) out[k] = bag_prof_entry{0, 0.0, 0.0, 0.0};
+  for (auto& r : ctx->prof) {
+    float ms = 0.f;
+    cudaEventElapsedTime(&ms, ctx->ev_pool[r.e0], ctx->ev_pool[r.e1]);
+    bag_prof_entry& o = out[r.kind];
+    o.launches += 1;
+    o.ms += ms;
+    o.flops += r.flops;
+    o.bytes += r.bytes;
+  }
+  if (stats) {
+    stats->T = ctx->T;
+    stats->B = ctx->B;
+    stats->nfe = nfe;
+    if (stats->mask)
+      for (int t = 0; t < ctx->T; ++t) stats->mask[t] = lg[(size_t)t * kLogFloats + 5] != 0.f;
+    if (stats->log) std::memcpy(stats->log, lg.data(), lg.size() * 4);
+  }
+  return s;
+}
+
 static bag_status check_device_error(bag_ctx* ctx) {
   DevState h;
   CK(cudaMemcpyAsync(&h, ctx->st, sizeof(h), cudaMemcpyDeviceToHost, ctx->stream));
@@ -1132,7 +1247,7 @@ static bag_status bag_gemm_bf16_impl(bag_ctx* ctx, const void* A, long lda, cons
 }
 
 static bag_status bag_attention_bf16_impl(bag_ctx* ctx, const void* q, const void* k, const void* v, void* o,
-                              long ld, int nq, int nk, int heads, int dh, int force_simt) {
+                              long ld, int nq, int nk, int heads, int dh, long vpad, int force_simt) {
   if (!ctx || !q || !k || !v || !o) return BAG_EINVAL;
   if (nq < 0 || nk <= 0 || heads <= 0 || (dh != 64 && dh != 128) || ld < (long)heads * dh)
     return fail(ctx, BAG_EINVAL, "bad attention shape");
@@ -1142,8 +1257,12 @@ static bag_status bag_attention_bf16_impl(bag_ctx* ctx, const void* q, const voi
   a.k = k;
   a.ldk = ld;
   a.v = v;
-  a.v_mode = 0;
+  a.v_mode = vpad > 0 ? 1 : 0;
   a.ldv = ld;
+  a.vpad = vpad;
+  if (vpad > 0 && (vpad < nk || vpad % 8)) return fail(ctx, BAG_EINVAL, "vpad must be >= nk and a multiple of 8");
+  if (!force_simt && !attention_tc_supported(a))
+    return fail(ctx, BAG_EUNSUPPORTED, "tensor-core attention needs dh 128, transposed V and 16-byte alignment");
   a.o = o;
   a.ldo = ld;
   a.nq = nq;
@@ -1245,6 +1364,7 @@ void bag_destroy(bag_ctx* ctx) {
   if (ctx->aarena) cudaFree(ctx->aarena);
   if (ctx->ev_in) cudaEventDestroy(ctx->ev_in);
   if (ctx->ev_out) cudaEventDestroy(ctx->ev_out);
+  for (auto ev : ctx->ev_pool) cudaEventDestroy(ev);
   if (ctx->stream) cudaStreamDestroy(ctx->stream);
   delete ctx;
 }
@@ -1351,6 +1471,13 @@ bag_status bag_forward_block(bag_ctx* ctx, int block, int t_mod, float* h) {
   return leave(ctx, bag_forward_block_impl(ctx, block, t_mod, h));
 }
 
+bag_status bag_profile_run(bag_ctx* ctx, float* x_inout, const bag_cond* cond, bag_stats* stats,
+                           bag_prof_entry* out) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, profile_run_impl(ctx, x_inout, cond, stats, out));
+}
+
 bag_status bag_launch_count(bag_ctx* ctx, long* out) {
   if (!ctx || !out) return BAG_EINVAL;
   *out = ctx->launches;
@@ -1366,10 +1493,10 @@ bag_status bag_gemm_bf16(bag_ctx* ctx, const void* A, long lda, const void* W, l
 }
 
 bag_status bag_attention_bf16(bag_ctx* ctx, const void* q, const void* k, const void* v, void* o,
-                              long ld, int nq, int nk, int heads, int dh, int force_simt) {
+                              long ld, int nq, int nk, int heads, int dh, long vpad, int force_simt) {
   if (!ctx) return BAG_EINVAL;
   CKS(enter(ctx));
-  return leave(ctx, bag_attention_bf16_impl(ctx, q, k, v, o, ld, nq, nk, heads, dh, force_simt));
+  return leave(ctx, bag_attention_bf16_impl(ctx, q, k, v, o, ld, nq, nk, heads, dh, vpad, force_simt));
 }
 
 bag_status bag_ln_mod(bag_ctx* ctx, const float* x, const float* shift, const float* scale, void* y,

@@ -23,6 +23,9 @@ Distributions (all exactly reproducible in IEEE fp32 on any machine):
 bf16 storage uses round-to-nearest-even of the fp32 value.
 """
 
+import concurrent.futures
+import os
+
 import numpy as np
 
 from .configs import TEMB_DIM
@@ -58,17 +61,52 @@ def normal_scale(std):
     return np.float32(float(std) * np.sqrt(3.0) / 65536.0)
 
 
-def normal(seed, key, n, std, offset=0, chunk=1 << 24):
+def _normal_range(out, s, c32, lo, hi, offset, chunk=1 << 16):
+    """Fill out[lo:hi] (cache-sized chunks, in-place ufuncs: numpy releases the GIL)."""
+    n = min(chunk, hi - lo)
+    base = np.arange(1, n + 1, dtype=np.uint64) * GOLDEN
+    z = np.empty(n, np.uint64)
+    t = np.empty(n, np.uint64)
+    q = np.empty(n, np.uint64)
+    m = np.uint64(0xFFFF)
+    with np.errstate(over="ignore"):
+        for a in range(lo, hi, chunk):
+            k = min(chunk, hi - a)
+            zz, tt, qq = z[:k], t[:k], q[:k]
+            np.add(base[:k], s + np.uint64(offset + a) * GOLDEN, out=zz)
+            np.right_shift(zz, np.uint64(30), out=tt)
+            np.bitwise_xor(zz, tt, out=zz)
+            np.multiply(zz, M1, out=zz)
+            np.right_shift(zz, np.uint64(27), out=tt)
+            np.bitwise_xor(zz, tt, out=zz)
+            np.multiply(zz, M2, out=zz)
+            np.right_shift(zz, np.uint64(31), out=tt)
+            np.bitwise_xor(zz, tt, out=zz)
+            np.bitwise_and(zz, m, out=qq)
+            for sh in (16, 32):
+                np.right_shift(zz, np.uint64(sh), out=tt)
+                np.bitwise_and(tt, m, out=tt)
+                np.add(qq, tt, out=qq)
+            np.right_shift(zz, np.uint64(48), out=tt)
+            np.add(qq, tt, out=qq)
+            o = out[a:a + k]
+            o[:] = qq.view(np.int64) - 131070
+            np.multiply(o, c32, out=o)
+
+
+def normal(seed, key, n, std, offset=0):
     """n fp32 samples of the Irwin-Hall(4) normal approximation with the given std."""
     out = np.empty(n, dtype=np.float32)
     c32 = normal_scale(std)
-    mask = np.uint64(0xFFFF)
-    for lo in range(0, n, chunk):
-        m = min(chunk, n - lo)
-        u = raw_u64(seed, key, m, offset + lo)
-        q = ((u & mask) + ((u >> np.uint64(16)) & mask) + ((u >> np.uint64(32)) & mask)
-             + (u >> np.uint64(48))).astype(np.int64) - 131070
-        out[lo:lo + m] = q.astype(np.float32) * c32
+    s = stream_start(seed, key)
+    nt = min(16, os.cpu_count() or 1) if n >= (1 << 22) else 1
+    if nt == 1:
+        _normal_range(out, s, c32, 0, n, offset)
+        return out
+    step = -(-n // nt)
+    with concurrent.futures.ThreadPoolExecutor(nt) as ex:
+        list(ex.map(lambda i: _normal_range(out, s, c32, i * step, min(n, (i + 1) * step), offset),
+                    range(nt)))
     return out
 
 
@@ -79,11 +117,27 @@ def uniform(seed, key, n, lo, hi):
 
 
 def bf16_round(x):
-    """Round fp32 values to the nearest bf16 (ties to even); returns fp32 values."""
-    x = np.ascontiguousarray(x, dtype=np.float32)
-    u = x.view(np.uint32).astype(np.uint64)
-    u = (u + np.uint64(0x7FFF) + ((u >> np.uint64(16)) & np.uint64(1))) & np.uint64(0xFFFF0000)
-    return u.astype(np.uint32).view(np.float32).reshape(x.shape)
+    """Round fp32 values to the nearest bf16 (ties to even); returns fp32 values.
+    (Finite inputs; the rounding carry may step into the exponent, as it should.)"""
+    x = np.array(x, dtype=np.float32, copy=True, order="C")
+    u = x.reshape(-1).view(np.uint32)
+    step = 1 << 18
+
+    def rnd(a):
+        v = u[a:a + step]
+        r = (v >> np.uint32(16)) & np.uint32(1)
+        r += np.uint32(0x7FFF)
+        v += r
+        v &= np.uint32(0xFFFF0000)
+
+    starts = range(0, u.size, step)
+    if u.size >= (1 << 22):
+        with concurrent.futures.ThreadPoolExecutor(min(16, os.cpu_count() or 1)) as ex:
+            list(ex.map(rnd, starts))
+    else:
+        for a in starts:
+            rnd(a)
+    return x
 
 
 def bf16_bits(x):

@@ -240,7 +240,13 @@ def test_attention_against_oracle(nq, nk, heads, dh, simt, lib):
     k, K_ = _bf16_tensor(12, (nk, d))
     v, V = _bf16_tensor(13, (nk, d))
     o = torch.zeros((nq, d), dtype=torch.bfloat16, device="cuda")
-    ctx.attention_bf16(Q, K_, V, o, nq, nk, heads, dh, simt)
+    if dh == 128:
+        vpad = (nk + 127) // 128 * 128
+        vt = torch.zeros((heads, dh, vpad), dtype=torch.bfloat16, device="cuda")
+        vt[:, :, :nk] = V.reshape(nk, heads, dh).permute(1, 2, 0)
+        ctx.attention_bf16(Q, K_, vt, o, nq, nk, heads, dh, vpad, simt)
+    else:
+        ctx.attention_bf16(Q, K_, V, o, nq, nk, heads, dh, 0, 1)
     torch.cuda.synchronize()
     rows = np.arange(nq) if nq <= 600 else np.r_[0:40, nq - 40:nq]
     ref = O.attention(q.reshape(nq, heads, dh).astype(np.float64),
