@@ -158,6 +158,129 @@ def oracle_s_per_sample(cfg, B, rep):
 
 
 # ---------------------------------------------------------------------------
+KERNEL_NAMES = {"gemm": "gemm_tc_kernel", "attention": "attn_tc_kernel",
+                "norm": "ln_mod_kernel", "signal": "ln_mod_kernel (signal)",
+                "gate": "gate_kernel", "cache": "cache_refresh/reuse_kernel"}
+KERNEL_SOURCES = {"gemm_tc_kernel": ["gemm.cu", "epilogue.cuh", "common.cuh"],
+                  "attn_tc_kernel": ["attn_tc.cu", "common.cuh"]}
+
+
+def source_sha1(kernel):
+    h = hashlib.sha1()
+    for f in KERNEL_SOURCES.get(kernel, []):
+        with open(os.path.join(ROOT, "paper_2608_09231_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def measured_traffic(kernel, shape):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the
+    current source of that kernel (else None)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        entries = json.load(f).get("entries", [])
+    for e in entries:
+        if (e.get("kernel") == kernel and list(e.get("shape", [])) == list(shape)
+                and e.get("source_sha1") == source_sha1(kernel)):
+            return e.get("dram_bytes_per_launch")
+    return None
+
+
+def dominant_roofline(recs, peaks, peak_src, cfg_name):
+    """Roofline of the (kernel, shape) group that takes the most event time."""
+    groups = {}
+    for r in recs:
+        key = (r["kind"], r["m"], r["n"], r["k"])
+        g = groups.setdefault(key, {"launches": 0, "ms": 0.0, "flops": 0.0, "bytes": 0.0})
+        g["launches"] += 1
+        g["ms"] += r["ms"]
+        g["flops"] += r["flops"]
+        g["bytes"] += r["bytes"]
+    kind, m, n, k = max(groups, key=lambda q: groups[q]["ms"])
+    g = groups[(kind, m, n, k)]
+    name = KERNEL_NAMES[kind]
+    avg_ms = g["ms"] / g["launches"]
+    total = sum(v["ms"] for v in groups.values())
+    shape = [m, n, k]
+    if g["flops"] > 0:
+        per = g["flops"] / g["launches"]
+        ach = per / (avg_ms * 1e-3) / 1e12
+        peak = peaks.get("bf16_tflops_sustained", 1700.0)
+        return {"bound": "tensor", "kernel": name, "shape": shape, "achieved": ach, "peak": peak,
+                "unit": "TFLOP/s", "frac": ach / peak, "traffic": measured_traffic(name, shape),
+                "peak_source": f"{peak_src} bf16 sustained (kernel timed inside the step)",
+                "launches": g["launches"], "avg_launch_ms": avg_ms, "flops_per_launch": per,
+                "share_of_profiled_time": g["ms"] / total}
+    per = g["bytes"] / g["launches"]
+    ach = per / (avg_ms * 1e-3) / 1e9
+    peak = peaks.get("hbm_gbs", 6800.0)
+    return {"bound": "hbm", "kernel": name, "shape": shape, "achieved": ach, "peak": peak,
+            "unit": "GB/s", "frac": ach / peak, "traffic": measured_traffic(name, shape),
+            "peak_source": f"{peak_src} HBM copy", "launches": g["launches"],
+            "avg_launch_ms": avg_ms, "bytes_per_launch": per,
+            "share_of_profiled_time": g["ms"] / total}
+
+
+def block_mode(args):
+    """One FLUX-shaped single-stream block forward (hidden 3072, 24 x 128 heads, MLP
+    12288, 4096 + 512 tokens) and the skip-path kernel: the per-block throughput of the
+    stack and the cost of a reused step.  Also the target of the ncu captures."""
+    import numpy as np
+    import torch
+
+    from paper_2608_09231_gb300 import bag, configs, synth
+
+    cfg = configs.get_config("flux_block")
+    d, F, N = cfg["hidden"], cfg["mlp"], cfg["n_img"] + cfg["n_txt"]
+    ctx = bag.create(cfg, T=cfg["T"], B=1)
+    stream = torch.cuda.current_stream()
+    ctx.set_stream(stream.cuda_stream)
+    inp = synth.make_inputs(cfg)
+    txt = torch.from_numpy(inp["txt"]).cuda().to(torch.bfloat16)
+    pooled = torch.from_numpy(inp["pooled"]).cuda()
+    ctx.prepare(txt, pooled)
+    h0 = torch.from_numpy(synth.normal(cfg["weight_seed"], 900, N * d, 1.0)).cuda().reshape(N, d)
+    h = h0.clone()
+    for _ in range(args.warmup):
+        ctx.forward_block(0, 0, h)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(True), torch.cuda.Event(True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        ctx.forward_block(0, 0, h)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    flops = 2.0 * N * d * (3 * d + F) + 2.0 * N * (d + F) * d + 4.0 * N * N * d
+    # skip path: h_out = h_in + R over the image stream
+    n = cfg["n_img"] * d
+    hin = h0[:cfg["n_img"]].contiguous()
+    R = torch.from_numpy(synth.normal(cfg["weight_seed"], 901, n, 0.3)).cuda()
+    out = torch.empty_like(hin)
+    for _ in range(3):
+        ctx.residual_add(out, hin, R, n)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(20):
+        ctx.residual_add(out, hin, R, n)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms_skip = e0.elapsed_time(e1) / 20
+    peaks, src = _peaks()
+    tf = flops / (ms * 1e-3) / 1e12
+    gbs = 12.0 * n / (ms_skip * 1e-3) / 1e9
+    print(json.dumps({"mode": "block", "workload": "FLUX-shaped single-stream block, 4096 img + "
+                      "512 txt tokens, d 3072, 24x128 heads, MLP 12288, bf16",
+                      "ms_per_block": ms, "block_tflops": tf,
+                      "frac_of_bf16_burst": tf / peaks.get("bf16_tflops", 1900.0),
+                      "skip_ms": ms_skip, "skip_gbs": gbs,
+                      "skip_frac_of_hbm": gbs / peaks.get("hbm_gbs", 6800.0),
+                      "peaks": src, "steps": args.steps, "warmup": args.warmup}))
+    ctx.close()
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -175,7 +298,11 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--mode", default="sample", choices=["sample", "block"])
     args = ap.parse_args()
+    if args.mode == "block":
+        block_mode(args)
+        return
     ws, rank, local = _dist()
 
     from paper_2608_09231_gb300 import configs
@@ -287,38 +414,30 @@ def main():
     h2d = x0.numel() * 4 + txth.numel() * 4 + pooledh.numel() * 4
     d2h = x0.numel() * 4 + T * (bag.LOG_FLOATS * 4 + 1) + 32
 
-    # profiled sample: per-kernel-class event timing (not part of the timed value)
+    # profiled sample: per-launch event timing (not part of the timed value)
     ctx.reset()
     x.copy_(x0)
     _, _, _, prof = ctx.profile_run(x, txt, pooled)
+    recs = ctx.profile_launches()
     peaks, peak_src = _peaks()
-    dom = max(prof, key=lambda k: prof[k]["ms"])
-    g = prof["gemm"]
+    peak_t = peaks.get("bf16_tflops_sustained", 1700.0)
+    roofline = dominant_roofline(recs, peaks, peak_src, args.config)
+    g, a = prof["gemm"], prof["attention"]
     gemm_tflops = g["flops"] / (g["ms"] * 1e-3) / 1e12 if g["ms"] > 0 else 0.0
-    a = prof["attention"]
     attn_tflops = a["flops"] / (a["ms"] * 1e-3) / 1e12 if a["ms"] > 0 else 0.0
     block_tflops = ((g["flops"] + a["flops"]) / ((g["ms"] + a["ms"]) * 1e-3) / 1e12
                     if g["ms"] + a["ms"] > 0 else 0.0)
-    peak_t = peaks.get("bf16_tflops_sustained", 1700.0)
-    traffic = None
-    tfile = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(tfile):
-        with open(tfile) as f:
-            tr = json.load(f)
-        src = open(os.path.join(ROOT, "paper_2608_09231_gb300", "csrc", "gemm.cu"), "rb").read()
-        if tr.get("gemm_cu_sha1") == hashlib.sha1(src).hexdigest() and tr.get("config") == args.config:
-            traffic = tr.get("gemm_bytes_per_launch")
-    roofline = {"bound": "tensor", "kernel": "gemm_tc_kernel (all block projections)",
-                "achieved": gemm_tflops, "peak": peak_t, "unit": "TFLOP/s",
-                "frac": gemm_tflops / peak_t, "traffic": traffic,
-                "peak_source": f"{peak_src} bf16 sustained",
-                "launches": g["launches"], "avg_launch_ms": g["ms"] / max(1, g["launches"]),
-                "flops_per_launch": g["flops"] / max(1, g["launches"])}
-    kernels = {k: {"launches": v["launches"], "ms": round(v["ms"], 3),
-                   "share": round(v["ms"] / max(1e-9, sum(p["ms"] for p in prof.values())), 4),
-                   **({"tflops": round(v["flops"] / (v["ms"] * 1e-3) / 1e12, 1)} if v["flops"] and v["ms"] else {}),
-                   **({"gbs": round(v["bytes"] / (v["ms"] * 1e-3) / 1e9, 1)} if not v["flops"] and v["ms"] else {})}
-               for k, v in prof.items()}
+    total_ms = sum(v["ms"] for v in prof.values())
+    kernels = {}
+    for k, v in prof.items():
+        e = {"launches": v["launches"], "ms": round(v["ms"], 3),
+             "share": round(v["ms"] / max(1e-9, total_ms), 4)}
+        if v["ms"] > 0:
+            if v["flops"]:
+                e["tflops"] = round(v["flops"] / (v["ms"] * 1e-3) / 1e12, 1)
+            else:
+                e["gbs"] = round(v["bytes"] / (v["ms"] * 1e-3) / 1e9, 1)
+        kernels[k] = e
 
     # budget sweep (context: how s/sample scales with B)
     sweep = {}

@@ -189,6 +189,16 @@ typedef struct {
 bag_status bag_profile_run(bag_ctx* ctx, float* x_inout, const bag_cond* cond, bag_stats* stats,
                            bag_prof_entry* out);
 
+/* Per-launch records of the last bag_profile_run: kind (BAG_PROF_*), shape (GEMM: M, N,
+ * K; attention: n_q, n_k, heads; 0 otherwise), event time, algorithmic flops and bytes.
+ * *n receives the number of records; up to max are copied to out (host; may be null). */
+typedef struct {
+  int kind, m, n, k;
+  float ms;
+  double flops, bytes;
+} bag_prof_launch;
+bag_status bag_profile_launches(bag_ctx* ctx, bag_prof_launch* out, long max, long* n);
+
 /* Number of kernel launches the last bag_run enqueued (graph nodes included). */
 bag_status bag_launch_count(bag_ctx* ctx, long* out);
 

@@ -27,7 +27,7 @@ EXPORTS = ["bag_create", "bag_destroy", "bag_last_error", "bag_set_stream", "bag
            "bag_set_policy", "bag_reset", "bag_step", "bag_run", "bag_run_host",
            "bag_get_weight", "bag_forward_block", "bag_prepare", "bag_launch_count",
            "bag_gemm_bf16", "bag_attention_bf16", "bag_ln_mod", "bag_residual_add",
-           "bag_profile_run"]
+           "bag_profile_run", "bag_profile_launches"]
 
 PROF_KINDS = ["gemm", "attention", "norm", "signal", "gate", "cache"]
 
@@ -53,6 +53,12 @@ class Cond(ctypes.Structure):
 
 class ProfEntry(ctypes.Structure):
     _fields_ = [("launches", ctypes.c_long), ("ms", ctypes.c_double), ("flops", ctypes.c_double),
+                ("bytes", ctypes.c_double)]
+
+
+class ProfLaunch(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int), ("m", ctypes.c_int), ("n", ctypes.c_int),
+                ("k", ctypes.c_int), ("ms", ctypes.c_float), ("flops", ctypes.c_double),
                 ("bytes", ctypes.c_double)]
 
 
@@ -98,6 +104,7 @@ def load(path=None):
         "bag_residual_add": ([_P, _P, _P, _P, _L], _I),
         "bag_profile_run": ([_P, _P, ctypes.POINTER(Cond), ctypes.POINTER(Stats),
                              ctypes.POINTER(ProfEntry)], _I),
+        "bag_profile_launches": ([_P, ctypes.POINTER(ProfLaunch), _L, ctypes.POINTER(_L)], _I),
     }
     for name, (args, res) in sig.items():
         f = getattr(lib, name)
@@ -206,6 +213,15 @@ class Context:
         prof = {k: dict(launches=out[i].launches, ms=out[i].ms, flops=out[i].flops,
                         bytes=out[i].bytes) for i, k in enumerate(PROF_KINDS)}
         return mask, log, s.nfe, prof
+
+    def profile_launches(self):
+        """Per-launch records of the last profile_run as a list of dicts."""
+        n = ctypes.c_long()
+        self._chk(self.lib.bag_profile_launches(self.h, None, 0, ctypes.byref(n)))
+        arr = (ProfLaunch * max(1, n.value))()
+        self._chk(self.lib.bag_profile_launches(self.h, arr, n.value, ctypes.byref(n)))
+        return [dict(kind=PROF_KINDS[r.kind], m=r.m, n=r.n, k=r.k, ms=r.ms, flops=r.flops,
+                     bytes=r.bytes) for r in arr[:n.value]]
 
     def run_host(self, x, txt, pooled):
         """All T steps with host numpy buffers (x updated in place); returns (mask, log, nfe)."""

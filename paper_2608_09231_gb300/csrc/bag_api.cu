@@ -11,6 +11,7 @@
 //   full   : text tokens -> stream, every block, R = h_out - h_in, m_last <- m_t
 //   reuse  : h_out = h_in + R
 //   suffix : final LN-mod + projection fused with the Euler update, t += 1
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -152,6 +153,7 @@ struct bag_ctx {
     int kind;
     double flops, bytes;
     int e0, e1;
+    int m, n, k;
   };
   std::vector<ProfRec> prof;
   std::vector<cudaEvent_t> ev_pool;
@@ -529,10 +531,10 @@ struct Enq {
   cudaStream_t s;
   long* count;
   cudaError_t e = cudaSuccess;
-  int pk = -1, pe0 = -1;
+  int pk = -1, pe0 = -1, pm = 0, pn = 0, pkk = 0;
   double pf = 0, pb = 0;
-  // announce the next launch (kind, algorithmic flops and bytes) for profiling
-  void pre(int kind, double flops, double bytes) {
+  // announce the next launch (kind, algorithmic flops and bytes, shape) for profiling
+  void pre(int kind, double flops, double bytes, int m = 0, int n = 0, int k = 0) {
     if (!ctx->profiling) return;
     pe0 = prof_event(ctx);
     if (pe0 < 0) return;
@@ -540,6 +542,9 @@ struct Enq {
     pk = kind;
     pf = flops;
     pb = bytes;
+    pm = m;
+    pn = n;
+    pkk = k;
   }
   void chk(cudaError_t r) {
     if (e == cudaSuccess && r != cudaSuccess) e = r;
@@ -548,7 +553,7 @@ struct Enq {
       const int pe1 = prof_event(ctx);
       if (pe1 >= 0) {
         cudaEventRecord(ctx->ev_pool[pe1], s);
-        ctx->prof.push_back({pk, pf, pb, pe0, pe1});
+        ctx->prof.push_back({pk, pf, pb, pe0, pe1, pm, pn, pkk});
       }
       pk = -1;
     }
@@ -574,7 +579,7 @@ static void enq_gemm(Enq& q, const void* A, long lda, const Tensor& W, long ldw,
     double out = (double)M * N * 4;
     if (e.kind == EPI_GATED_RES || e.kind == EPI_RES_ADD) out = (double)M * N * 8;
     else if (e.kind == EPI_QKV || e.kind == EPI_GELU) out = (double)M * N * es;
-    q.pre(BAG_PROF_GEMM, 2.0 * M * N * K, ((double)M + N) * K * es + out);
+    q.pre(BAG_PROF_GEMM, 2.0 * M * N * K, ((double)M + N) * K * es + out, M, N, K);
   }
   q.chk(gemm(A, lda, W.p, ldw, M, N, K, q.ctx->act_bf16, e, q.ctx->st ? &q.ctx->st->err : nullptr, q.s));
 }
@@ -641,7 +646,7 @@ static void enq_attn(Enq& q, const void* Q, const void* K, const void* V, long v
   a.st = st;
   a.flag_want = flag_want;
   q.pre(BAG_PROF_ATTN, 4.0 * nq * nk * ctx->H * ctx->dh,
-        ((double)nq * 2 + 2.0 * nk) * ctx->d * ctx->act_size);
+        ((double)nq * 2 + 2.0 * nk) * ctx->d * ctx->act_size, nq, nk, ctx->H);
   q.chk(attention(a, ctx->st ? &ctx->st->err : nullptr, q.s));
 }
 
@@ -1261,8 +1266,6 @@ static bag_status bag_attention_bf16_impl(bag_ctx* ctx, const void* q, const voi
   a.ldv = ld;
   a.vpad = vpad;
   if (vpad > 0 && (vpad < nk || vpad % 8)) return fail(ctx, BAG_EINVAL, "vpad must be >= nk and a multiple of 8");
-  if (!force_simt && !attention_tc_supported(a))
-    return fail(ctx, BAG_EUNSUPPORTED, "tensor-core attention needs dh 128, transposed V and 16-byte alignment");
   a.o = o;
   a.ldo = ld;
   a.nq = nq;
@@ -1272,6 +1275,8 @@ static bag_status bag_attention_bf16_impl(bag_ctx* ctx, const void* q, const voi
   a.bf16 = 1;
   a.st = nullptr;
   a.flag_want = -1;
+  if (!force_simt && !attention_tc_supported(a))
+    return fail(ctx, BAG_EUNSUPPORTED, "tensor-core attention needs dh 128, transposed V and 16-byte alignment");
   CK(attention(a, &ctx->st_op->err, ctx->stream, force_simt));
   return BAG_OK;
 }
@@ -1476,6 +1481,20 @@ bag_status bag_profile_run(bag_ctx* ctx, float* x_inout, const bag_cond* cond, b
   if (!ctx) return BAG_EINVAL;
   CKS(enter(ctx));
   return leave(ctx, profile_run_impl(ctx, x_inout, cond, stats, out));
+}
+
+bag_status bag_profile_launches(bag_ctx* ctx, bag_prof_launch* out, long max, long* n) {
+  if (!ctx || !n) return BAG_EINVAL;
+  *n = (long)ctx->prof.size();
+  if (!out) return BAG_OK;
+  const long m = std::min<long>(max, (long)ctx->prof.size());
+  for (long i = 0; i < m; ++i) {
+    const auto& r = ctx->prof[i];
+    float ms = 0.f;
+    cudaEventElapsedTime(&ms, ctx->ev_pool[r.e0], ctx->ev_pool[r.e1]);
+    out[i] = bag_prof_launch{r.kind, r.m, r.n, r.k, ms, r.flops, r.bytes};
+  }
+  return BAG_OK;
 }
 
 bag_status bag_launch_count(bag_ctx* ctx, long* out) {
