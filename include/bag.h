@@ -225,6 +225,14 @@ bag_status bag_attention_bf16(bag_ctx* ctx, const void* q, const void* k, const 
 bag_status bag_ln_mod(bag_ctx* ctx, const float* x, const float* shift, const float* scale,
                       void* y, int rows, int cols);
 
+/* Trajectory signal of Eq. 3 with the L1 norm: relative change sum|a - b| / sum|b| of
+ * two device tensors a, b [rows, cols] (dtype BAG_F32 or BAG_BF16; b is the reference).
+ * scratch: caller-owned device fp32 [2 * rows] for per-row partial sums (overwritten);
+ * out: device fp32 [3] receives {sum|a-b| / sum|b|, sum|a-b|, sum|b|}.  The row
+ * partials are summed in a fixed order, so repeated calls give identical results. */
+bag_status bag_rel_l1(bag_ctx* ctx, const void* a, const void* b, int dtype, long rows,
+                      long cols, float* scratch, float* out);
+
 /* Skip path (plain residual reuse): out = h_in + R, fp32 device, n elements (n % 4 == 0). */
 bag_status bag_residual_add(bag_ctx* ctx, float* out, const float* h_in, const float* R, long n);
 

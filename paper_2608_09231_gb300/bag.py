@@ -27,7 +27,7 @@ EXPORTS = ["bag_create", "bag_destroy", "bag_last_error", "bag_set_stream", "bag
            "bag_set_policy", "bag_reset", "bag_step", "bag_run", "bag_run_host",
            "bag_get_weight", "bag_forward_block", "bag_prepare", "bag_launch_count",
            "bag_gemm_bf16", "bag_attention_bf16", "bag_ln_mod", "bag_residual_add",
-           "bag_profile_run", "bag_profile_launches"]
+           "bag_profile_run", "bag_profile_launches", "bag_rel_l1"]
 
 PROF_KINDS = ["gemm", "attention", "norm", "signal", "gate", "cache"]
 
@@ -102,6 +102,7 @@ def load(path=None):
         "bag_attention_bf16": ([_P, _P, _P, _P, _P, _L, _I, _I, _I, _I, _L, _I], _I),
         "bag_ln_mod": ([_P, _P, _P, _P, _P, _I, _I], _I),
         "bag_residual_add": ([_P, _P, _P, _P, _L], _I),
+        "bag_rel_l1": ([_P, _P, _P, _I, _L, _L, _P, _P], _I),
         "bag_profile_run": ([_P, _P, ctypes.POINTER(Cond), ctypes.POINTER(Stats),
                              ctypes.POINTER(ProfEntry)], _I),
         "bag_profile_launches": ([_P, ctypes.POINTER(ProfLaunch), _L, ctypes.POINTER(_L)], _I),
@@ -262,6 +263,11 @@ class Context:
     def ln_mod(self, x, shift, scale, y, rows, cols):
         self._chk(self.lib.bag_ln_mod(self.h, _ptr(x), _ptr(shift), _ptr(scale), _ptr(y), rows,
                                       cols))
+
+    def rel_l1(self, a, b, rows, cols, scratch, out, bf16=None):
+        dt = (1 if a.dtype.itemsize == 2 else 0) if bf16 is None else int(bf16)
+        self._chk(self.lib.bag_rel_l1(self.h, _ptr(a), _ptr(b), dt, rows, cols, _ptr(scratch),
+                                      _ptr(out)))
 
     def residual_add(self, out, h_in, R, n):
         self._chk(self.lib.bag_residual_add(self.h, _ptr(out), _ptr(h_in), _ptr(R), n))

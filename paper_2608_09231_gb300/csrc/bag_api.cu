@@ -1302,6 +1302,16 @@ static bag_status bag_ln_mod_impl(bag_ctx* ctx, const float* x, const float* shi
   return BAG_OK;
 }
 
+static bag_status bag_rel_l1_impl(bag_ctx* ctx, const void* a, const void* b, int dtype, long rows,
+                                   long cols, float* scratch, float* out) {
+  if (!a || !b || !scratch || !out) return fail(ctx, BAG_EINVAL, "null pointer");
+  if (rows <= 0 || cols <= 0 || (dtype != BAG_F32 && dtype != BAG_BF16))
+    return fail(ctx, BAG_EINVAL, "bad rel_l1 shape or dtype");
+  CK(rel_l1_partials(a, b, dtype == BAG_BF16, rows, cols, scratch, ctx->stream));
+  CK(rel_l1_finalize(scratch, rows, out, ctx->stream));
+  return BAG_OK;
+}
+
 static bag_status bag_residual_add_impl(bag_ctx* ctx, float* out, const float* h_in, const float* R, long n) {
   if (!ctx || !out || !h_in || !R) return BAG_EINVAL;
   if (n < 0 || n % 4) return fail(ctx, BAG_EINVAL, "n must be a multiple of 4");
@@ -1523,6 +1533,13 @@ bag_status bag_ln_mod(bag_ctx* ctx, const float* x, const float* shift, const fl
   if (!ctx) return BAG_EINVAL;
   CKS(enter(ctx));
   return leave(ctx, bag_ln_mod_impl(ctx, x, shift, scale, y, rows, cols));
+}
+
+bag_status bag_rel_l1(bag_ctx* ctx, const void* a, const void* b, int dtype, long rows, long cols,
+                      float* scratch, float* out) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, bag_rel_l1_impl(ctx, a, b, dtype, rows, cols, scratch, out));
 }
 
 bag_status bag_residual_add(bag_ctx* ctx, float* out, const float* h_in, const float* R, long n) {

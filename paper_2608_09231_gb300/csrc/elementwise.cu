@@ -184,6 +184,32 @@ cudaError_t rel_l1_partials(const void* a, const void* b, int a_bf16, long rows,
   return cudaGetLastError();
 }
 
+// out[0] = sum(num) / sum(den), out[1] = sum(num), out[2] = sum(den) over the per-row
+// partials, summed in the same fixed order as the gate kernel's drift reduction.
+__global__ void rel_l1_finalize_kernel(const float* partial, long rows, float* out) {
+  const int lane = threadIdx.x;
+  float num = 0.f, den = 0.f;
+  for (long r = lane; r < rows; r += 32) {
+    num += partial[2 * r];
+    den += partial[2 * r + 1];
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    num += __shfl_xor_sync(0xffffffffu, num, off);
+    den += __shfl_xor_sync(0xffffffffu, den, off);
+  }
+  if (lane == 0) {
+    out[0] = __fdiv_rn(num, den);
+    out[1] = num;
+    out[2] = den;
+  }
+}
+
+cudaError_t rel_l1_finalize(const float* partial, long rows, float* out, cudaStream_t s) {
+  rel_l1_finalize_kernel<<<1, 32, 0, s>>>(partial, rows, out);
+  return cudaGetLastError();
+}
+
 // ---------------------------------------------------------------------------
 // gate + pacing (one warp)
 // ---------------------------------------------------------------------------

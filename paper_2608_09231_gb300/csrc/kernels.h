@@ -140,6 +140,7 @@ cudaError_t fill_synth(void* dst, long n, uint64_t seed, uint64_t key, float c32
 cudaError_t residual_add(float* out, const float* a, const float* b, long n, cudaStream_t s);
 cudaError_t rel_l1_partials(const void* a, const void* b, int a_bf16, long rows, long cols,
                             float* partial, cudaStream_t s);
+cudaError_t rel_l1_finalize(const float* partial, long rows, float* out, cudaStream_t s);
 
 // one-time kernel attribute setup (dynamic shared memory limits); call before capture
 cudaError_t kernels_init();

@@ -218,6 +218,31 @@ def test_ln_mod_against_oracle(rows, cols, lib):
     ctx.close()
 
 
+@pytest.mark.parametrize("rows,cols,bf16", [(4096, 3072, 1), (37, 256, 0), (1, 64, 1)])
+def test_rel_l1_against_oracle(rows, cols, bf16, lib):
+    ctx = bag.create("tiny", T=2, B=1)
+    a = synth.normal(21, 1, rows * cols, 1.0).reshape(rows, cols)
+    b = a + synth.normal(21, 2, rows * cols, 0.05).reshape(rows, cols)
+    if bf16:
+        a, b = synth.bf16_round(a), synth.bf16_round(b)
+    dt = torch.bfloat16 if bf16 else torch.float32
+    A = torch.from_numpy(a).cuda().to(dt)
+    Bt = torch.from_numpy(b).cuda().to(dt)
+    scratch = torch.empty(2 * rows, dtype=torch.float32, device="cuda")
+    out = torch.empty(3, dtype=torch.float32, device="cuda")
+    ctx.rel_l1(A, Bt, rows, cols, scratch, out)
+    torch.cuda.synchronize()
+    ref = O.rel_l1(a.astype(np.float64), b.astype(np.float64))
+    got = out.cpu().numpy()
+    assert abs(float(got[0]) - ref) <= 1e-5 * ref
+    assert abs(float(got[2]) - np.abs(b.astype(np.float64)).sum()) <= 1e-5 * float(got[2])
+    # identical inputs give exactly zero
+    ctx.rel_l1(Bt, Bt, rows, cols, scratch, out)
+    torch.cuda.synchronize()
+    assert float(out[0].item()) == 0.0
+    ctx.close()
+
+
 def test_residual_add_exact(lib):
     ctx = bag.create("tiny", T=2, B=1)
     n = 1 << 20
