@@ -233,6 +233,21 @@ bag_status bag_ln_mod(bag_ctx* ctx, const float* x, const float* shift, const fl
 bag_status bag_rel_l1(bag_ctx* ctx, const void* a, const void* b, int dtype, long rows,
                       long cols, float* scratch, float* out);
 
+/* Allocation-free bag_rel_l1 (the paper has no counterpart: this is a deployment
+ * variant).  For callers that cannot call cudaMalloc - code inside a framework whose
+ * caching allocator owns the device memory, or loops that cannot take cudaMalloc's
+ * implicit synchronisation - and so cannot create a context either: no context, no
+ * allocation.  a, b: device [rows, cols] (dtype BAG_F32 or BAG_BF16); out: device fp32
+ * [3] as for bag_rel_l1; work runs on cuda_stream (a cudaStream_t, null = legacy).
+ * The row partials live in a fixed file-scope device array of 2 * 65536 floats held by
+ * every GPU that loads the library until exit: rows > 65536 returns BAG_EINVAL.  The
+ * first call on a device looks the array's address up (cudaGetSymbolAddress) and
+ * should come before any stream capture.  All calls share the array and it keeps the
+ * last call's contents (each call writes what it reads); calls that overlap on the GPU
+ * race.  Errors are reported through bag_last_error(NULL). */
+bag_status bag_rel_l1_noalloc(const void* a, const void* b, int dtype, long rows, long cols,
+                              float* out, void* cuda_stream);
+
 /* Skip path (plain residual reuse): out = h_in + R, fp32 device, n elements (n % 4 == 0). */
 bag_status bag_residual_add(bag_ctx* ctx, float* out, const float* h_in, const float* R, long n);
 

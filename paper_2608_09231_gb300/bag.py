@@ -27,7 +27,7 @@ EXPORTS = ["bag_create", "bag_destroy", "bag_last_error", "bag_set_stream", "bag
            "bag_set_policy", "bag_reset", "bag_step", "bag_run", "bag_run_host",
            "bag_get_weight", "bag_forward_block", "bag_prepare", "bag_launch_count",
            "bag_gemm_bf16", "bag_attention_bf16", "bag_ln_mod", "bag_residual_add",
-           "bag_profile_run", "bag_profile_launches", "bag_rel_l1"]
+           "bag_profile_run", "bag_profile_launches", "bag_rel_l1", "bag_rel_l1_noalloc"]
 
 PROF_KINDS = ["gemm", "attention", "norm", "signal", "gate", "cache"]
 
@@ -103,6 +103,7 @@ def load(path=None):
         "bag_ln_mod": ([_P, _P, _P, _P, _P, _I, _I], _I),
         "bag_residual_add": ([_P, _P, _P, _P, _L], _I),
         "bag_rel_l1": ([_P, _P, _P, _I, _L, _L, _P, _P], _I),
+        "bag_rel_l1_noalloc": ([_P, _P, _I, _L, _L, _P, _P], _I),
         "bag_profile_run": ([_P, _P, ctypes.POINTER(Cond), ctypes.POINTER(Stats),
                              ctypes.POINTER(ProfEntry)], _I),
         "bag_profile_launches": ([_P, ctypes.POINTER(ProfLaunch), _L, ctypes.POINTER(_L)], _I),
@@ -271,6 +272,17 @@ class Context:
 
     def residual_add(self, out, h_in, R, n):
         self._chk(self.lib.bag_residual_add(self.h, _ptr(out), _ptr(h_in), _ptr(R), n))
+
+
+def rel_l1_noalloc(a, b, rows, cols, out, stream=0, bf16=None):
+    """bag_rel_l1_noalloc: the signal reduction with no context and no allocation
+    (scratch in a fixed device array of the library; see include/bag.h)."""
+    lib = load()
+    dt = (1 if a.dtype.itemsize == 2 else 0) if bf16 is None else int(bf16)
+    st = lib.bag_rel_l1_noalloc(_ptr(a), _ptr(b), dt, rows, cols, _ptr(out),
+                                ctypes.c_void_p(stream))
+    if st != 0:
+        raise BagError(st, lib.bag_last_error(None).decode())
 
 
 def create(cfg_or_name, T=None, B=None, tau=0.5, **overrides):

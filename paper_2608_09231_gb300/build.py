@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libbag.so")
 
-SOURCES = ["bag_api.cu", "gemm.cu", "attn.cu", "attn_tc.cu", "elementwise.cu"]
+SOURCES = ["bag_api.cu", "gemm.cu", "attn.cu", "attn_tc.cu", "elementwise.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -163,6 +163,8 @@ struct bag_ctx {
 
 static std::string g_create_error;
 
+void bag::set_global_error(const std::string& msg) { g_create_error = msg; }
+
 #define CK(expr)                                                                     \
   do {                                                                               \
     cudaError_t _e = (expr);                                                         \

@@ -142,6 +142,12 @@ cudaError_t rel_l1_partials(const void* a, const void* b, int a_bf16, long rows,
                             float* partial, cudaStream_t s);
 cudaError_t rel_l1_finalize(const float* partial, long rows, float* out, cudaStream_t s);
 
+// message returned by bag_last_error(NULL) (entry points without a context)
+}  // namespace bag
+#include <string>
+namespace bag {
+void set_global_error(const std::string& msg);
+
 // one-time kernel attribute setup (dynamic shared memory limits); call before capture
 cudaError_t kernels_init();
 
