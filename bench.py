@@ -281,6 +281,33 @@ def block_mode(args):
     ctx.close()
 
 
+def profile_mode(args):
+    """One profiled sample (direct launches, only the taken branch launched) and its
+    per-kernel-class split; the process an ncu launch list is taken on, because ncu
+    does not profile kernels inside graphs that hold conditional nodes."""
+    import torch
+
+    from paper_2608_09231_gb300 import bag, configs, synth
+
+    cfg = configs.get_config(args.config)
+    T = args.T or cfg["T"]
+    ctx = bag.create(cfg, T=T, B=args.budget)
+    inp = synth.make_inputs(cfg)
+    x = torch.from_numpy(inp["x"]).cuda()
+    txt = torch.from_numpy(inp["txt"]).cuda()
+    if cfg["dtype"] == "bf16":
+        txt = txt.to(torch.bfloat16)
+    pooled = torch.from_numpy(inp["pooled"]).cuda()
+    mask, _, nfe, prof = ctx.profile_run(x, txt, pooled)
+    torch.cuda.synchronize()
+    tot = sum(v["ms"] for v in prof.values())
+    print(json.dumps({"mode": "profile", "config": args.config, "T": T, "B": args.budget,
+                      "nfe": nfe, "mask": [int(m) for m in mask],
+                      "kernels": {k: {"launches": v["launches"], "ms": round(v["ms"], 3),
+                                      "share": round(v["ms"] / tot, 4)} for k, v in prof.items()}}))
+    ctx.close()
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -298,10 +325,14 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
-    ap.add_argument("--mode", default="sample", choices=["sample", "block"])
+    ap.add_argument("--mode", default="sample", choices=["sample", "block", "profile"])
+    ap.add_argument("--T", type=int, default=0, help="profile mode: override the step count")
     args = ap.parse_args()
     if args.mode == "block":
         block_mode(args)
+        return
+    if args.mode == "profile":
+        profile_mode(args)
         return
     ws, rank, local = _dist()
 
