@@ -185,9 +185,12 @@ def _mlp(x, wu, bu, wd, bd):
     return linear(gelu_tanh(linear(x, wu, bu)), wd, bd)
 
 
-def double_block(img, txt, mod_img, mod_txt, W, ang, H):
+def double_block(img, txt, mod_img, mod_txt, W, ang, H, rows=None):
     """Double-stream (MMDiT) block: separate weights per stream, joint attention over
-    [txt; img].  mod_* = (shift1, scale1, gate1, shift2, scale2, gate2)."""
+    [txt; img].  mod_* = (shift1, scale1, gate1, shift2, scale2, gate2).
+
+    rows: optional joint-sequence rows (text first) at which to evaluate the outputs;
+    then the return value is the joint output [len(rows), d] at those rows only."""
     d = img.shape[1]
     nx = txt.shape[0]
 
@@ -201,6 +204,18 @@ def double_block(img, txt, mod_img, mod_txt, W, ang, H):
     q = apply_rope(_heads(qkv[:, :d], H), ang)
     k = apply_rope(_heads(qkv[:, d:2 * d], H), ang)
     v = _heads(qkv[:, 2 * d:], H)
+    if rows is not None:
+        rows = np.asarray(rows)
+        a = attention(q, k, v, q_rows=rows).reshape(-1, d)
+        hj = np.concatenate([txt, img], axis=0)[rows]
+        out = np.empty_like(hj)
+        for sel, pre, m in ((rows < nx, "txt", mt), (rows >= nx, "img", mi)):
+            if not sel.any():
+                continue
+            x = hj[sel] + m[2] * linear(a[sel], W[pre + "_proj_w"], W[pre + "_proj_b"])
+            out[sel] = x + m[5] * _mlp(modulate(layer_norm(x), m[3], m[4]), W[pre + "_up_w"],
+                                       W[pre + "_up_b"], W[pre + "_down_w"], W[pre + "_down_b"])
+        return out
     a = attention(q, k, v).reshape(-1, d)
     a_t, a_i = a[:nx], a[nx:]
     img = img + mi[2] * linear(a_i, W["img_proj_w"], W["img_proj_b"])
@@ -212,17 +227,21 @@ def double_block(img, txt, mod_img, mod_txt, W, ang, H):
     return img, txt
 
 
-def wan_block(x, ctx, e, W, ang, H):
+def wan_block(x, ctx, e, W, ang, H, rows=None):
     """Wan-style block: modulated self-attention with 3D RoPE, cross-attention to the
     text context (plain LayerNorm on the query side, no gate), modulated GELU FFN.
-    e = (shift1, scale1, gate1, shift2, scale2, gate2)."""
+    e = (shift1, scale1, gate1, shift2, scale2, gate2).
+    rows: optional image rows at which to evaluate (then only those rows are returned)."""
     d = x.shape[1]
     ch = [e[i * d:(i + 1) * d] for i in range(6)]
     qkv = linear(modulate(layer_norm(x), ch[0], ch[1]), W["sa_qkv_w"], W["sa_qkv_b"])
     q = apply_rope(_heads(qkv[:, :d], H), ang)
     k = apply_rope(_heads(qkv[:, d:2 * d], H), ang)
     v = _heads(qkv[:, 2 * d:], H)
-    x = x + ch[2] * linear(attention(q, k, v).reshape(-1, d), W["sa_o_w"], W["sa_o_b"])
+    if rows is not None:
+        rows = np.asarray(rows)
+        x = x[rows]
+    x = x + ch[2] * linear(attention(q, k, v, q_rows=rows).reshape(-1, d), W["sa_o_w"], W["sa_o_b"])
     qc = _heads(linear(layer_norm(x), W["ca_q_w"], W["ca_q_b"]), H)
     kv = linear(ctx, W["ca_kv_w"], W["ca_kv_b"])
     kc, vc = _heads(kv[:, :d], H), _heads(kv[:, d:], H)
@@ -443,10 +462,10 @@ def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=Non
     return {"x": x, "mask": mask, "log": log, "nfe": c}
 
 
-def forward_block(cfg, W, block_index, h_joint, vec, rows=None):
-    """One block of the stack applied to a given joint stream (text rows first for the
-    MMDiT kinds; image rows only for Wan, with txt the context).  Used to check a single
-    block at full width on sampled rows."""
+def forward_block(cfg, W, block_index, h_joint, vec, rows=None, txt=None):
+    """One block of the stack applied to a given stream: the joint [txt; img] sequence
+    (text rows first) for single- and double-stream blocks, the image stream for Wan
+    blocks (txt = the cross-attention context).  rows: evaluate only those rows."""
     W = to64(W)
     G, blk = W["global"], W["blocks"][block_index]
     H = cfg["heads"]
@@ -454,4 +473,10 @@ def forward_block(cfg, W, block_index, h_joint, vec, rows=None):
     mod = block_modulation(cfg, G, blk, vec)
     if blk["type"] == "single":
         return single_block(h_joint, mod, blk, ang, H, rows=rows)
-    raise NotImplementedError(blk["type"])
+    if blk["type"] == "double":
+        nx = cfg["n_txt"]
+        out = double_block(h_joint[nx:], h_joint[:nx], mod[0], mod[1], blk, ang, H, rows=rows)
+        if rows is None:
+            return np.concatenate([out[1], out[0]], axis=0)
+        return out
+    return wan_block(h_joint, txt, mod, blk, ang, H, rows=rows)

@@ -129,7 +129,8 @@ struct bag_ctx {
   float* pooled_stage = nullptr;
   float2* rope = nullptr;
   float* dsig = nullptr;
-  void *sin_all = nullptr, *t1o = nullptr, *svec = nullptr;
+  float *sin_all = nullptr, *t1o = nullptr, *svec = nullptr;  // fp32 conditioning chain
+  __nv_bfloat16* splitbuf = nullptr;  // [T, 2 * max(256, d)] hi|lo halves (bf16 configs)
   float *vec_all = nullptr, *mod_all = nullptr, *wan_shared = nullptr;
   DevState* st = nullptr;     // sampler state
   DevState* st_op = nullptr;  // state for single-operation calls
@@ -487,9 +488,10 @@ static bag_status alloc_activations(bag_ctx* ctx) {
   A.add((void**)&ctx->pooled_stage, (size_t)d * 4);
   A.add((void**)&ctx->rope, (size_t)ctx->nrope * (ctx->dh / 2) * sizeof(float2));
   A.add((void**)&ctx->dsig, (size_t)T * 4);
-  A.add(&ctx->sin_all, (size_t)T * kTembDim * es);
-  A.add(&ctx->t1o, (size_t)T * d * es);
-  A.add(&ctx->svec, (size_t)T * d * es);
+  A.add((void**)&ctx->sin_all, (size_t)T * kTembDim * 4);
+  A.add((void**)&ctx->t1o, (size_t)T * d * 4);
+  A.add((void**)&ctx->svec, (size_t)T * d * 4);
+  A.add((void**)&ctx->splitbuf, (size_t)T * 2 * std::max<long>(kTembDim, d) * 2);
   A.add((void**)&ctx->vec_all, (size_t)T * d * 4);
   A.add((void**)&ctx->mod_all, (size_t)T * ctx->mod_stride * 4);
   if (wan) A.add((void**)&ctx->wan_shared, (size_t)T * 8 * d * 4);
@@ -902,14 +904,28 @@ static bag_status enq_prepare(bag_ctx* ctx, const bag_cond* cond) {
     CK(cudaMemcpyAsync(ctx->pooled_stage, cond->pooled, (size_t)d * 4, cudaMemcpyDeviceToDevice, s));
   long cnt = 0;
   Enq q{ctx, s, &cnt};
-  q.chk(sinusoid_all(ctx->sin_all, ctx->act_bf16, ctx->T, kTembDim, s));
+  // The conditioning chain stays fp32: for bf16 configs each GEMM takes its fp32
+  // activation as bf16 hi + lo halves (split A), so the modulation vectors carry no
+  // bf16 rounding of the activations (an error that would be the same for every token
+  // and every block and so would not average out).
+  const int bf = ctx->act_bf16;
+  auto gemm_f32_act = [&](const float* act, int K, const Tensor& W, int N, const Epi& e) {
+    if (bf) {
+      q.chk(split_bf16(ctx->splitbuf, act, ctx->T, K, s));
+      q.pre(BAG_PROF_GEMM, 4.0 * ctx->T * N * K, (double)N * K * 2, ctx->T, N, 2 * K);
+      q.chk(gemm(ctx->splitbuf, 2L * K, W.p, K, ctx->T, N, K, 1, e, &ctx->st->err, s, 0, 1));
+    } else {
+      enq_gemm(q, act, K, W, K, ctx->T, N, K, e);
+    }
+  };
+  q.chk(sinusoid_all(ctx->sin_all, 0, ctx->T, kTembDim, s));
   Epi e1 = base_epi(ctx, nullptr, -1);
   e1.kind = EPI_SILU;
   e1.bias = (const float*)ctx->G.at("t1_b").p;
   e1.out = ctx->t1o;
   e1.ldo = d;
-  e1.out_bf16 = ctx->act_bf16;
-  enq_gemm(q, ctx->sin_all, kTembDim, ctx->G.at("t1_w"), kTembDim, ctx->T, (int)d, kTembDim, e1);
+  e1.out_bf16 = 0;
+  gemm_f32_act(ctx->sin_all, kTembDim, ctx->G.at("t1_w"), (int)d, e1);
   Epi e2 = base_epi(ctx, nullptr, -1);
   e2.kind = EPI_VEC;
   e2.bias = (const float*)ctx->G.at("t2_b").p;
@@ -918,8 +934,8 @@ static bag_status enq_prepare(bag_ctx* ctx, const bag_cond* cond) {
   e2.addend = ctx->arch.kind == BAG_KIND_WAN ? nullptr : ctx->pooled_stage;
   e2.out2 = ctx->svec;
   e2.ldo2 = d;
-  e2.out2_bf16 = ctx->act_bf16;
-  enq_gemm(q, ctx->t1o, d, ctx->G.at("t2_w"), d, ctx->T, (int)d, (int)d, e2);
+  e2.out2_bf16 = 0;
+  gemm_f32_act(ctx->t1o, (int)d, ctx->G.at("t2_w"), (int)d, e2);
   Epi e3 = base_epi(ctx, nullptr, -1);
   e3.kind = EPI_STORE;
   e3.bias = ctx->bmod;
@@ -927,12 +943,12 @@ static bag_status enq_prepare(bag_ctx* ctx, const bag_cond* cond) {
   if (ctx->arch.kind == BAG_KIND_WAN) {
     e3.out = ctx->wan_shared;
     e3.ldo = 8 * d;
-    enq_gemm(q, ctx->svec, d, ctx->wmod, d, ctx->T, (int)ctx->n_mod, (int)d, e3);
+    gemm_f32_act(ctx->svec, (int)d, ctx->wmod, (int)ctx->n_mod, e3);
     q.chk(expand_wan_mod(ctx->mod_all, ctx->wan_shared, ctx->wan_tabs, ctx->T, ctx->nblk, (int)d, s));
   } else {
     e3.out = ctx->mod_all;
     e3.ldo = ctx->mod_stride;
-    enq_gemm(q, ctx->svec, d, ctx->wmod, d, ctx->T, (int)ctx->n_mod, (int)d, e3);
+    gemm_f32_act(ctx->svec, (int)d, ctx->wmod, (int)ctx->n_mod, e3);
   }
   if (q.e != cudaSuccess) return fail(ctx, BAG_ECUDA, std::string("prepare: ") + cudaGetErrorString(q.e));
   ctx->n_prepare = cnt;

@@ -434,6 +434,23 @@ cudaError_t expand_wan_mod(float* mod_all, const float* shared8d, const float* t
   return cudaGetLastError();
 }
 
+__global__ void split_bf16_kernel(__nv_bfloat16* dst, const float* src, long rows, long cols) {
+  const long n = rows * cols;
+  for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
+    const long r = i / cols, c = i % cols;
+    const float x = src[i];
+    const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+    dst[r * 2 * cols + c] = hi;
+    dst[r * 2 * cols + cols + c] = __float2bfloat16_rn(x - __bfloat162float(hi));
+  }
+}
+
+cudaError_t split_bf16(__nv_bfloat16* dst, const float* src, long rows, long cols, cudaStream_t s) {
+  if (rows * cols <= 0) return cudaSuccess;
+  split_bf16_kernel<<<grid_for(rows * cols, 256), 256, 0, s>>>(dst, src, rows, cols);
+  return cudaGetLastError();
+}
+
 __global__ void to_bf16_kernel(__nv_bfloat16* dst, const float* src, long n) {
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x)
     dst[i] = __float2bfloat16_rn(src[i]);

@@ -138,7 +138,7 @@ struct TcCfg {
 template <int BN>
 __global__ void __launch_bounds__(192, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const Epi e, int M, int N, int K, int* err) {
+                   const Epi e, int M, int N, int K, int a_split, int* err) {
   using C = TcCfg<BN>;
   if (epi_skip(e.st, e.flag_want)) return;
   extern __shared__ uint8_t smem_raw[];
@@ -156,7 +156,10 @@ __global__ void __launch_bounds__(192, 1)
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int num_m = (M + TC_BM - 1) / TC_BM, num_n = N / BN;
-  const int tiles = num_m * num_n, kit = K / TC_BK;
+  // a_split: A holds [hi | lo] bf16 halves of an fp32 activation ([M, 2K]); the K loop
+  // runs twice as long, feeding each W chunk once with hi and once with lo, so the
+  // product is accurate to fp32 accumulation while W is streamed once.
+  const int tiles = num_m * num_n, kit = (a_split ? 2 : 1) * (K / TC_BK);
   const int t = epi_step(e);
 
   if (threadIdx.x == 0) {
@@ -200,8 +203,10 @@ __global__ void __launch_bounds__(192, 1)
             break;
           }
           mbar_arrive_expect_tx(full + s, C::STAGE_BYTES);
-          tma_load_2d(sA + s * C::A_BYTES, &tmA, kb * TC_BK, mt * TC_BM, full + s);
-          tma_load_2d(sB + s * C::B_BYTES, &tmB, kb * TC_BK, nt * BN, full + s);
+          const int ka = a_split ? (kb & 1) * K + (kb >> 1) * TC_BK : kb * TC_BK;
+          const int kw = a_split ? (kb >> 1) * TC_BK : kb * TC_BK;
+          tma_load_2d(sA + s * C::A_BYTES, &tmA, ka, mt * TC_BM, full + s);
+          tma_load_2d(sB + s * C::B_BYTES, &tmB, kw, nt * BN, full + s);
           ++issued;
           if (++s == C::STAGES) {
             s = 0;
@@ -301,15 +306,15 @@ __global__ void __launch_bounds__(192, 1)
 
 template <int BN>
 static cudaError_t launch_tc(const void* A, long lda, const void* W, long ldw, int M, int N,
-                             int K, const Epi& e, int* err, cudaStream_t s) {
+                             int K, const Epi& e, int* err, cudaStream_t s, int a_split) {
   using C = TcCfg<BN>;
   CUtensorMap ta, tb;
-  if (encode_tmap_2d_bf16(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)lda * 2, TC_BK, TC_BM) ||
+  if (encode_tmap_2d_bf16(&ta, A, (uint64_t)K * (a_split ? 2 : 1), (uint64_t)M, (uint64_t)lda * 2, TC_BK, TC_BM) ||
       encode_tmap_2d_bf16(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)ldw * 2, TC_BK, BN))
     return cudaErrorInvalidValue;
   const int tiles = ((M + TC_BM - 1) / TC_BM) * (N / BN);
   const int grid = std::min(tiles, num_sms());
-  gemm_tc_kernel<BN><<<grid, 192, C::SMEM, s>>>(ta, tb, e, M, N, K, err);
+  gemm_tc_kernel<BN><<<grid, 192, C::SMEM, s>>>(ta, tb, e, M, N, K, a_split, err);
   return cudaGetLastError();
 }
 
@@ -336,7 +341,8 @@ int gemm_tc_supported(int M, int N, int K, long lda, long ldw) {
 }
 
 cudaError_t gemm(const void* A, long lda, const void* W, long ldw, int M, int N, int K,
-                 int in_bf16, const Epi& epi_in, int* err, cudaStream_t s, int force_simt) {
+                 int in_bf16, const Epi& epi_in, int* err, cudaStream_t s, int force_simt,
+                 int a_split) {
   if (M <= 0 || N <= 0) return cudaSuccess;
   Epi e = epi_in;
   e.M = M;
@@ -346,12 +352,14 @@ cudaError_t gemm(const void* A, long lda, const void* W, long ldw, int M, int N,
     // bf16 operands always take the tensor-core path; a shape or pointer it cannot
     // tile is an error, never a silent switch to the CUDA-core kernel
     if (!aligned || !gemm_tc_supported(M, N, K, lda, ldw)) return cudaErrorNotSupported;
+    if (a_split && lda < 2L * K) return cudaErrorInvalidValue;
     const int ns = num_sms();
     const int mt = (M + TC_BM - 1) / TC_BM;
-    if (N % 256 == 0 && mt * (N / 256) >= ns) return launch_tc<256>(A, lda, W, ldw, M, N, K, e, err, s);
-    if (N % 128 == 0 && mt * (N / 128) >= ns) return launch_tc<128>(A, lda, W, ldw, M, N, K, e, err, s);
-    return launch_tc<64>(A, lda, W, ldw, M, N, K, e, err, s);
+    if (N % 256 == 0 && mt * (N / 256) >= ns) return launch_tc<256>(A, lda, W, ldw, M, N, K, e, err, s, a_split);
+    if (N % 128 == 0 && mt * (N / 128) >= ns) return launch_tc<128>(A, lda, W, ldw, M, N, K, e, err, s, a_split);
+    return launch_tc<64>(A, lda, W, ldw, M, N, K, e, err, s, a_split);
   }
+  if (a_split) return cudaErrorInvalidValue;
   if (N % 4 != 0) return cudaErrorInvalidValue;
   dim3 grid((N + 63) / 64, (M + 63) / 64);
   if (in_bf16)

@@ -87,8 +87,13 @@ struct Epi {
 // C[M,N] = A[M,K] W[N,K]^T with the fused epilogue.  Tensor-core path for bf16
 // operands; fp32 operands (and shapes the tensor-core path does not tile) go to the
 // CUDA-core path.
+// a_split (bf16 only): A is [M, 2K] = [hi | lo] bf16 halves of an fp32 activation
+// (see split_bf16); the product then carries fp32-level accuracy in A.
 cudaError_t gemm(const void* A, long lda, const void* W, long ldw, int M, int N, int K,
-                 int in_bf16, const Epi& epi, int* err, cudaStream_t s, int force_simt = 0);
+                 int in_bf16, const Epi& epi, int* err, cudaStream_t s, int force_simt = 0,
+                 int a_split = 0);
+// dst [rows, 2*cols] bf16 = [bf16(x) | bf16(x - bf16(x))] of src fp32 [rows, cols]
+cudaError_t split_bf16(__nv_bfloat16* dst, const float* src, long rows, long cols, cudaStream_t s);
 int gemm_tc_supported(int M, int N, int K, long lda, long ldw);
 
 struct AttnArgs {

@@ -418,6 +418,27 @@ def test_wan_block_brute_force():
     assert np.allclose(got, want, atol=1e-12)
 
 
+def test_row_restricted_blocks_equal_full_evaluation():
+    """Evaluating a block at a subset of rows gives those rows of the full evaluation."""
+    rng = np.random.default_rng(8)
+    d, H, F, ni, nx = 8, 2, 12, 5, 3
+    Wd = _rand_block(rng, synth.block_shapes({"hidden": d, "mlp": F}, "double"))
+    img, txt = rng.normal(size=(ni, d)), rng.normal(size=(nx, d))
+    mi, mt = rng.normal(size=6 * d) * 0.5, rng.normal(size=6 * d) * 0.5
+    ang = O.rope_angles(np.concatenate([np.zeros((nx, 3)), rng.integers(0, 4, size=(ni, 3))]),
+                        (0, 2, 2))
+    gi, gt = O.double_block(img, txt, mi, mt, Wd, ang, H)
+    full = np.concatenate([gt, gi])
+    rows = [6, 0, 2, 4]
+    assert np.allclose(O.double_block(img, txt, mi, mt, Wd, ang, H, rows=rows), full[rows],
+                       atol=1e-13)
+    Ww = _rand_block(rng, synth.block_shapes({"hidden": d, "mlp": F}, "wan"))
+    e = rng.normal(size=6 * d) * 0.5
+    angw = O.rope_angles(rng.integers(0, 4, size=(ni, 3)).astype(float), (2, 0, 2))
+    fw = O.wan_block(img, txt, e, Ww, angw, H)
+    assert np.allclose(O.wan_block(img, txt, e, Ww, angw, H, rows=[3, 1]), fw[[3, 1]], atol=1e-13)
+
+
 def test_zero_gate_blocks_are_identity():
     rng = np.random.default_rng(6)
     d, H, F = 8, 2, 12
