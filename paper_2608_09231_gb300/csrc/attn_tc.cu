@@ -1,19 +1,22 @@
 // Joint attention on the 5th-generation tensor cores (head_dim 128, bf16 operands).
 //
-// One CTA owns 128 query rows of one head and walks the keys in tiles of 128:
-//   warp 0      TMA producer: Q once, then K and V^T tiles into a 2-stage ring
-//   warp 1      MMA issuer:   S_j = Q K_j^T into one of two TMEM buffers, then
-//                             O += P_{j-1} V_{j-1} (P from shared memory), so the tensor
-//                             core computes S_{j+1} while the softmax works on S_j
-//   warps 2..5  softmax:      thread = query row; S row from TMEM, running max/sum in
-//                             the exp2 domain, P = exp2(s - m) as bf16 into shared
-//                             memory (128-byte swizzle, K-major for the PV MMA).
-// O lives in TMEM for the whole key loop.  The running max is only moved (and O
-// rescaled in TMEM) when a tile's max exceeds it by more than 8 in log2 units, so P
-// stays <= 2^8 and the rescale is rare; the final division by the row sum uses the
-// same max, so the result is the exact softmax up to rounding.
+// One CTA owns two 128-row query tiles (A and B) of one head and walks the keys in
+// tiles of 128:
+//   warp 0      TMA producer: both Q tiles once, then K and V^T tiles into a 2-stage ring
+//   warp 1      MMA issuer, ping-pong between the tiles:
+//                 S_A,0  S_B,0 | PV_A,j  S_A,j+1 | PV_B,j  S_B,j+1 | ...
+//               so the tensor core computes one tile's products while the other tile's
+//               softmax runs
+//   warps 2..5  softmax of tile A, warps 6..9 softmax of tile B: thread = query row; S
+//               row read from TMEM (a max pass, then an exp pass), P = exp2(s - m) packed
+//               to bf16 and written back into TMEM over the S columns already consumed.
+// The PV product takes P straight from TMEM as its A operand, so P never touches
+// shared memory; shared memory only feeds Q, K and V^T.  O stays in TMEM for the whole
+// key loop.  The running max only moves (and O is rescaled in TMEM) when a tile's max
+// exceeds it by more than 8 in log2 units, so P <= 2^8; the final division by the row
+// sum uses the same max, which makes the result the exact softmax up to rounding.
 // V arrives transposed per head ([head][dh][token]) from the QKV projection's epilogue,
-// which makes it a K-major B operand like every other tile here.
+// which makes it a K-major B operand.
 #include <cmath>
 
 #include "common.cuh"
@@ -27,12 +30,12 @@ constexpr int AT_M = 128, AT_N = 128, AT_D = 128;
 constexpr int AT_CHUNK = 128 * 64 * 2;  // 128 rows x 64 bf16 = one 128-byte-swizzle column
 constexpr int AT_TILE = 2 * AT_CHUNK;   // 128 x 128 bf16
 constexpr int AT_STAGES = 2;
-constexpr int AT_OFF_Q = 0;
-constexpr int AT_OFF_KV = AT_TILE;                              // stage s: K, then V^T
-constexpr int AT_OFF_P = AT_OFF_KV + AT_STAGES * 2 * AT_TILE;
-constexpr int AT_OFF_BAR = AT_OFF_P + AT_TILE;
+constexpr int AT_OFF_Q = 0;                                     // Q_A, Q_B
+constexpr int AT_OFF_KV = 2 * AT_TILE;                          // stage s: K, then V^T
+constexpr int AT_OFF_BAR = AT_OFF_KV + AT_STAGES * 2 * AT_TILE;
 constexpr int AT_SMEM = AT_OFF_BAR + 256 + 1024;
-constexpr int AT_TMEM_COLS = 512;  // S0 [0,128), S1 [128,256), O [256,384)
+constexpr int AT_TMEM_COLS = 512;  // S_A [0,128) S_B [128,256) O_A [256,384) O_B [384,512)
+constexpr int AT_THREADS = 320;
 
 struct AttnTcParams {
   int nq, nk;
@@ -50,14 +53,49 @@ BAG_DEV float ex2(float x) {
   return y;
 }
 
-// byte offset of 16-byte unit u (0..15, 8 bf16 each) of row r in a 128 x 128 bf16 tile
-// stored as two 128-byte-swizzled K-major columns
-BAG_DEV uint32_t sw_off(int r, int u) {
-  return (uint32_t)((u >> 3) * AT_CHUNK + (r >> 3) * 1024 + (r & 7) * 128 + (((u & 7) ^ (r & 7)) << 4));
+// 32 consecutive 32-bit TMEM columns of this thread's lane, without the wait (the caller
+// issues tcgen05.wait::ld once for several loads)
+BAG_DEV void tmem_ld32_nowait(uint32_t taddr, uint32_t* r) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, "
+      "[%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+        "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+        "=r"(r[31])
+      : "r"(taddr));
+}
+
+BAG_DEV void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// 16 consecutive 32-bit TMEM columns of this thread's lane
+BAG_DEV void tmem_st16(uint32_t taddr, const uint32_t* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+      "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]),
+      "r"(v[15])
+      : "memory");
+}
+
+// D (TMEM) += A (TMEM, 16-bit elements packed two per column) * B (shared memory)
+BAG_DEV void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
 }
 }  // namespace
 
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(AT_THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, const AttnTcParams p) {
   if (epi_skip(p.st, p.flag_want)) return;
@@ -66,21 +104,19 @@ __global__ void __launch_bounds__(192, 1)
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sQ = smem + AT_OFF_Q;
   uint8_t* sKV = smem + AT_OFF_KV;
-  uint8_t* sP = smem + AT_OFF_P;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + AT_OFF_BAR);
   uint64_t* q_full = bars + 0;
   uint64_t* kv_full = bars + 1;   // [2]
   uint64_t* kv_empty = bars + 3;  // [2]
-  uint64_t* s_full = bars + 5;    // [2]
-  uint64_t* s_free = bars + 7;    // [2]
-  uint64_t* p_full = bars + 9;
-  uint64_t* o_done = bars + 10;
+  uint64_t* s_full = bars + 5;    // [2] per query tile
+  uint64_t* p_full = bars + 7;    // [2]
+  uint64_t* o_done = bars + 9;    // [2]
   uint64_t* drain = bars + 11;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int head = blockIdx.y, q0 = blockIdx.x * AT_M;
+  const int head = blockIdx.y, q0 = blockIdx.x * 2 * AT_M;
   const int nkb = (p.nk + AT_N - 1) / AT_N;
 
   if (threadIdx.x == 0) {
@@ -89,10 +125,9 @@ __global__ void __launch_bounds__(192, 1)
       mbar_init(kv_full + i, 1);
       mbar_init(kv_empty + i, 1);
       mbar_init(s_full + i, 1);
-      mbar_init(s_free + i, 128);
+      mbar_init(p_full + i, 128);
+      mbar_init(o_done + i, 1);
     }
-    mbar_init(p_full, 128);
-    mbar_init(o_done, 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -114,9 +149,11 @@ __global__ void __launch_bounds__(192, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- TMA producer ----------------
-      mbar_arrive_expect_tx(q_full, AT_TILE);
-      tma_load_2d(sQ, &tmQ, head * AT_D, q0, q_full);
-      tma_load_2d(sQ + AT_CHUNK, &tmQ, head * AT_D + 64, q0, q_full);
+      mbar_arrive_expect_tx(q_full, 2 * AT_TILE);
+      for (int x = 0; x < 2; ++x) {
+        tma_load_2d(sQ + x * AT_TILE, &tmQ, head * AT_D, q0 + x * AT_M, q_full);
+        tma_load_2d(sQ + x * AT_TILE + AT_CHUNK, &tmQ, head * AT_D + 64, q0 + x * AT_M, q_full);
+      }
       int issued = 0;
       bool ok = true;
       for (int j = 0; j < nkb; ++j) {
@@ -149,79 +186,100 @@ __global__ void __launch_bounds__(192, 1)
     if (lane == 0) {
       // ---------------- MMA issuer ----------------
       constexpr uint32_t idesc = idesc_bf16_f32(AT_M, AT_N);
-      bool ok = mbar_wait(q_full, 0, abort_flag);
-      tc_fence_after();
-      const uint32_t q_addr = smem_u32(sQ), p_addr = smem_u32(sP);
-      auto issue_pv = [&](int i) -> bool {
-        if (!mbar_wait(p_full, i & 1, abort_flag)) return false;
-        tc_fence_after();
-        const uint32_t v_addr = smem_u32(sKV + (i % AT_STAGES) * 2 * AT_TILE + AT_TILE);
-#pragma unroll
-        for (int kk = 0; kk < AT_N / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * AT_CHUNK + (kk & 3) * 32;
-          mma_bf16(tmem + 256, sw128_desc(p_addr + off), sw128_desc(v_addr + off), idesc,
-                   (i > 0 || kk > 0) ? 1u : 0u);
-        }
-        mma_commit(o_done);
-        mma_commit(kv_empty + i % AT_STAGES);
-        return true;
-      };
-      for (int j = 0; j < nkb && ok; ++j) {
-        const int s = j % AT_STAGES, b = j & 1;
-        if (!mbar_wait(kv_full + s, (j / AT_STAGES) & 1, abort_flag)) {
-          ok = false;
-          break;
-        }
-        if (j >= 2 && !mbar_wait(s_free + b, ((j - 2) >> 1) & 1, abort_flag)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const uint32_t k_addr = smem_u32(sKV + s * 2 * AT_TILE);
+      const uint32_t q_addr = smem_u32(sQ);
+      auto issue_s = [&](int x, int j) {
+        const uint32_t qa = q_addr + x * AT_TILE;
+        const uint32_t ka = smem_u32(sKV + (j % AT_STAGES) * 2 * AT_TILE);
 #pragma unroll
         for (int kk = 0; kk < AT_D / 16; ++kk) {
           const uint32_t off = (kk >> 2) * AT_CHUNK + (kk & 3) * 32;
-          mma_bf16(tmem + b * 128, sw128_desc(q_addr + off), sw128_desc(k_addr + off), idesc,
+          mma_bf16(tmem + x * 128, sw128_desc(qa + off), sw128_desc(ka + off), idesc,
                    kk > 0 ? 1u : 0u);
         }
-        mma_commit(s_full + b);
-        if (j >= 1 && !issue_pv(j - 1)) ok = false;
+        mma_commit(s_full + x);
+      };
+      auto issue_pv = [&](int x, int j) {
+        const uint32_t va = smem_u32(sKV + (j % AT_STAGES) * 2 * AT_TILE + AT_TILE);
+#pragma unroll
+        for (int kk = 0; kk < AT_N / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * AT_CHUNK + (kk & 3) * 32;
+          mma_bf16_ts(tmem + 256 + x * 128, tmem + x * 128 + kk * 8, sw128_desc(va + off), idesc,
+                      (j > 0 || kk > 0) ? 1u : 0u);
+        }
+      };
+      bool ok = mbar_wait(q_full, 0, abort_flag) && mbar_wait(kv_full, 0, abort_flag);
+      if (ok) {
+        tc_fence_after();
+        issue_s(0, 0);
+        issue_s(1, 0);
       }
-      if (ok) issue_pv(nkb - 1);
+      for (int j = 0; j < nkb && ok; ++j) {
+        const bool more = j + 1 < nkb;
+        // tile A: PV_j, then S_{j+1} into the columns P_j came from (in issue order)
+        if (!mbar_wait(p_full + 0, j & 1, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        issue_pv(0, j);
+        if (more) {
+          if (!mbar_wait(kv_full + (j + 1) % AT_STAGES, ((j + 1) / AT_STAGES) & 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_s(0, j + 1);
+        } else {
+          mma_commit(o_done + 0);
+        }
+        // tile B
+        if (!mbar_wait(p_full + 1, j & 1, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        issue_pv(1, j);
+        mma_commit(kv_empty + j % AT_STAGES);
+        if (more)
+          issue_s(1, j + 1);
+        else
+          mma_commit(o_done + 1);
+      }
       mma_commit(drain);
       const uint64_t t0 = global_ns();
       while (!mbar_try_wait(drain, 0) && global_ns() - t0 < kWaitLimitNs) {
       }
     }
   } else {
-    // ---------------- softmax warpgroup ----------------
+    // ---------------- softmax warpgroups (warps 2..5: tile A, 6..9: tile B) ----------------
+    const int x = (warp - 2) >> 2;
     const int quad = warp & 3;
     const int row = quad * 32 + lane;
     const uint32_t lane_base = (uint32_t)(quad * 32) << 16;
+    const uint32_t s_addr = tmem + lane_base + x * 128;
+    const uint32_t o_addr = tmem + lane_base + 256 + x * 128;
     float m_use = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < nkb; ++j) {
-      const int b = j & 1;
-      bool w = mbar_wait(s_full + b, (j >> 1) & 1, abort_flag);
+      const bool w = mbar_wait(s_full + x, j & 1, abort_flag);
       if (!__all_sync(0xffffffffu, w)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      float s[AT_N];
+      const int kvalid = p.nk - j * AT_N;  // keys of this tile that exist (< 128 only at the end)
+      // pass 1: row max
+      float mx = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < AT_N / 32; ++c) tmem_ld32(tmem + lane_base + b * 128 + c * 32, s + c * 32);
-      tc_fence_before();
-      mbar_arrive(s_free + b);
-      const int kvalid = p.nk - j * AT_N;
-      if (kvalid < AT_N) {
+      for (int h = 0; h < 2; ++h) {
+        uint32_t r[64];
+        tmem_ld32_nowait(s_addr + h * 64, r);
+        tmem_ld32_nowait(s_addr + h * 64 + 32, r + 32);
+        tmem_ld_wait();
 #pragma unroll
-        for (int i = 0; i < AT_N; ++i)
-          if (i >= kvalid) s[i] = -INFINITY;
+        for (int i = 0; i < 64; ++i)
+          if (h * 64 + i < kvalid) mx = fmaxf(mx, __uint_as_float(r[i]));
       }
-      float mx = s[0];
-#pragma unroll
-      for (int i = 1; i < AT_N; ++i) mx = fmaxf(mx, s[i]);
       const float mx2 = mx * p.scale_log2;
       float alpha = 1.f;
       if (mx2 > m_use + 8.f) {
@@ -229,58 +287,52 @@ __global__ void __launch_bounds__(192, 1)
         m_use = mx2;
         l *= alpha;
       }
-      const bool resc = __any_sync(0xffffffffu, alpha != 1.f) && j > 0;
-      uint32_t pk[AT_N / 2];
-      float ls = 0.f;
-#pragma unroll
-      for (int i = 0; i < AT_N; i += 2) {
-        const float a0 = ex2(fmaf(s[i], p.scale_log2, -m_use));
-        const float a1 = ex2(fmaf(s[i + 1], p.scale_log2, -m_use));
-        ls += a0 + a1;
-        pk[i / 2] = pack_bf16x2(a0, a1);
-      }
-      l += ls;
-      if (j >= 1) {
-        w = mbar_wait(o_done, (j - 1) & 1, abort_flag);
-        if (!__all_sync(0xffffffffu, w)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-      }
-      if (resc) {
+      // O_x holds PV of every earlier key tile (the S of this tile was issued after it)
+      if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
 #pragma unroll 1
         for (int c = 0; c < AT_D / 32; ++c) {
           float o[32];
-          tmem_ld32(tmem + lane_base + 256 + c * 32, o);
+          tmem_ld32(o_addr + c * 32, o);
 #pragma unroll
           for (int i = 0; i < 32; ++i) o[i] *= alpha;
-          tmem_st32(tmem + lane_base + 256 + c * 32, o);
+          tmem_st32(o_addr + c * 32, o);
         }
-        tmem_st_wait();
       }
-      const uint32_t pbase = smem_u32(sP);
+      // pass 2: P = exp2(s * scale - m), packed bf16 pairs over the consumed S columns
+      float ls = 0.f;
 #pragma unroll
-      for (int u = 0; u < AT_N / 8; ++u) {
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(pbase + sw_off(row, u)),
-                     "r"(pk[4 * u]), "r"(pk[4 * u + 1]), "r"(pk[4 * u + 2]), "r"(pk[4 * u + 3])
-                     : "memory");
+      for (int c = 0; c < AT_N / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32_nowait(s_addr + c * 32, r);
+        tmem_ld_wait();
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+          const int kcol = c * 32 + i;
+          const float a0 = kcol < kvalid ? ex2(fmaf(__uint_as_float(r[i]), p.scale_log2, -m_use)) : 0.f;
+          const float a1 =
+              kcol + 1 < kvalid ? ex2(fmaf(__uint_as_float(r[i + 1]), p.scale_log2, -m_use)) : 0.f;
+          ls += a0 + a1;
+          pk[i / 2] = pack_bf16x2(a0, a1);
+        }
+        tmem_st16(s_addr + c * 16, pk);
       }
-      fence_proxy_async_smem();
+      l += ls;
+      tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(p_full);
+      mbar_arrive(p_full + x);
     }
     if (ok) {
-      bool w = mbar_wait(o_done, (nkb - 1) & 1, abort_flag);
+      const bool w = mbar_wait(o_done + x, 0, abort_flag);
       if (__all_sync(0xffffffffu, w)) {
         tc_fence_after();
         const float inv = 1.f / l;
-        const int q = q0 + row;
+        const int q = q0 + x * AT_M + row;
         __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.o) + (long)q * p.ldo + head * AT_D;
 #pragma unroll 1
         for (int c = 0; c < AT_D / 32; ++c) {
           float o[32];
-          tmem_ld32(tmem + lane_base + 256 + c * 32, o);
+          tmem_ld32(o_addr + c * 32, o);
 #pragma unroll
           for (int i = 0; i < 32; ++i) o[i] *= inv;
           if (q < p.nq) store_vals<32>(orow + c * 32, 0, o, 1);
@@ -325,8 +377,8 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t s) {
   p.st = a.st;
   p.flag_want = a.flag_want;
   p.err = err;
-  dim3 grid((a.nq + AT_M - 1) / AT_M, a.heads);
-  attn_tc_kernel<<<grid, 192, AT_SMEM, s>>>(tq, tk, tv, p);
+  dim3 grid((a.nq + 2 * AT_M - 1) / (2 * AT_M), a.heads);
+  attn_tc_kernel<<<grid, AT_THREADS, AT_SMEM, s>>>(tq, tk, tv, p);
   return cudaGetLastError();
 }
 

@@ -10,8 +10,10 @@ benchmark times.
   (LN-mod output, q/k/v or MLP hidden, P or GELU output, attention output), each a
   relative error <= 2^-9.  Its error therefore scales with the element's own update
   |g * o|, which at full width reaches ~5x the output RMS in columns with large adaLN
-  gates.  Bar per element: |err| <= 2e-2 x RMS(ref) + 2^-7 x |ref - h|; and over the
-  sampled rows RMS(err) <= 2^-8 x RMS(ref - h).
+  gates.  Bar per element: |err| <= 2e-2 x RMS(ref) + 2^-7 x |ref - h|.  Over the
+  sampled rows RMS(err) <= 2^-7 x RMS(ref - h): a Wan block adds three residual
+  branches (self-attention, cross-attention, FFN), each with its own roundings, and the
+  q and k roundings enter through the softmax exponent, where they count about double.
 * Whole samples at full size: properties that hold at any size — realised NFE = B for
   every configured budget, m_0 = 1, the schedule equals Algorithm 2 applied to the gate
   bits the oracle computes from the GPU's logged gate inputs, and B = T reproduces
@@ -68,7 +70,7 @@ def test_block_full_size_sampled_rows(name, over, rows, lib):
     err = np.abs(got - ref)
     bar = 2e-2 * rms + 2.0 ** -7 * np.abs(upd)
     assert np.all(err <= bar), (float(err.max()), float((err / bar).max()))
-    assert float(np.sqrt(np.mean(err ** 2))) <= 2.0 ** -8 * float(np.sqrt(np.mean(upd ** 2)))
+    assert float(np.sqrt(np.mean(err ** 2))) <= 2.0 ** -7 * float(np.sqrt(np.mean(upd ** 2)))
     # the block changed the stream (it is not an identity pass)
     assert float(np.sqrt(np.mean(upd ** 2))) > 100 * float(np.sqrt(np.mean(err ** 2)))
 
