@@ -8,8 +8,8 @@
 //               so the tensor core computes one tile's products while the other tile's
 //               softmax runs
 //   warps 2..5  softmax of tile A, warps 6..9 softmax of tile B: thread = query row; S
-//               row read from TMEM (a max pass, then an exp pass), P = exp2(s - m) packed
-//               to bf16 and written back into TMEM over the S columns already consumed.
+//               row read from TMEM into registers in one round trip, P = exp2(s - m)
+//               packed to bf16 and written back into TMEM over the S columns.
 // The PV product takes P straight from TMEM as its A operand, so P never touches
 // shared memory; shared memory only feeds Q, K and V^T.  O stays in TMEM for the whole
 // key loop.  The running max only moves (and O is rescaled in TMEM) when a tile's max
@@ -268,18 +268,19 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       }
       tc_fence_after();
       const int kvalid = p.nk - j * AT_N;  // keys of this tile that exist (< 128 only at the end)
-      // pass 1: row max
-      float mx = -INFINITY;
+      // the whole S row in registers: four loads, one wait
+      uint32_t r[AT_N];
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        uint32_t r[64];
-        tmem_ld32_nowait(s_addr + h * 64, r);
-        tmem_ld32_nowait(s_addr + h * 64 + 32, r + 32);
-        tmem_ld_wait();
+      for (int c = 0; c < AT_N / 32; ++c) tmem_ld32_nowait(s_addr + c * 32, r + c * 32);
+      tmem_ld_wait();
+      if (kvalid < AT_N) {
 #pragma unroll
-        for (int i = 0; i < 64; ++i)
-          if (h * 64 + i < kvalid) mx = fmaxf(mx, __uint_as_float(r[i]));
+        for (int i = 0; i < AT_N; ++i)
+          if (i >= kvalid) r[i] = __float_as_uint(-INFINITY);
       }
+      float mx = __uint_as_float(r[0]);
+#pragma unroll
+      for (int i = 1; i < AT_N; ++i) mx = fmaxf(mx, __uint_as_float(r[i]));
       const float mx2 = mx * p.scale_log2;
       float alpha = 1.f;
       if (mx2 > m_use + 8.f) {
@@ -287,7 +288,24 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         m_use = mx2;
         l *= alpha;
       }
-      // O_x holds PV of every earlier key tile (the S of this tile was issued after it)
+      // P = exp2(s * scale - m) (masked keys give exp2(-inf) = 0), packed bf16 pairs
+      // written over the S columns already read
+      float ls = 0.f;
+#pragma unroll
+      for (int c = 0; c < AT_N / 32; ++c) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+          const float a0 = ex2(fmaf(__uint_as_float(r[c * 32 + i]), p.scale_log2, -m_use));
+          const float a1 = ex2(fmaf(__uint_as_float(r[c * 32 + i + 1]), p.scale_log2, -m_use));
+          ls += a0 + a1;
+          pk[i / 2] = pack_bf16x2(a0, a1);
+        }
+        tmem_st16(s_addr + c * 16, pk);
+      }
+      l += ls;
+      // O_x holds PV of every earlier key tile (the S of this tile was issued after it);
+      // rescale it before this tile's PV is issued
       if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
 #pragma unroll 1
         for (int c = 0; c < AT_D / 32; ++c) {
@@ -298,26 +316,6 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
           tmem_st32(o_addr + c * 32, o);
         }
       }
-      // pass 2: P = exp2(s * scale - m), packed bf16 pairs over the consumed S columns
-      float ls = 0.f;
-#pragma unroll
-      for (int c = 0; c < AT_N / 32; ++c) {
-        uint32_t r[32];
-        tmem_ld32_nowait(s_addr + c * 32, r);
-        tmem_ld_wait();
-        uint32_t pk[16];
-#pragma unroll
-        for (int i = 0; i < 32; i += 2) {
-          const int kcol = c * 32 + i;
-          const float a0 = kcol < kvalid ? ex2(fmaf(__uint_as_float(r[i]), p.scale_log2, -m_use)) : 0.f;
-          const float a1 =
-              kcol + 1 < kvalid ? ex2(fmaf(__uint_as_float(r[i + 1]), p.scale_log2, -m_use)) : 0.f;
-          ls += a0 + a1;
-          pk[i / 2] = pack_bf16x2(a0, a1);
-        }
-        tmem_st16(s_addr + c * 16, pk);
-      }
-      l += ls;
       tmem_st_wait();
       tc_fence_before();
       mbar_arrive(p_full + x);
