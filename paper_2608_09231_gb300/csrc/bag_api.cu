@@ -588,6 +588,26 @@ static void enq_gemm(Enq& q, const void* A, long lda, const Tensor& W, long ldw,
   q.chk(gemm(A, lda, W.p, ldw, M, N, K, q.ctx->act_bf16, e, q.ctx->st ? &q.ctx->st->err : nullptr, q.s));
 }
 
+// Two projections with the same N and K (image and text stream of a double-stream
+// block) in one tensor-core launch; fp32 configurations run them one after the other.
+static void enq_gemm2(Enq& q, const void* A0, long lda0, const Tensor& W0, long ldw0, int M0,
+                      const Epi& e0, const void* A1, long lda1, const Tensor& W1, long ldw1,
+                      int M1, const Epi& e1, int N, int K) {
+  if (!q.ctx->act_bf16) {
+    enq_gemm(q, A0, lda0, W0, ldw0, M0, N, K, e0);
+    enq_gemm(q, A1, lda1, W1, ldw1, M1, N, K, e1);
+    return;
+  }
+  const double es = 2.0;
+  double out = (double)(M0 + M1) * N * 4;
+  if (e0.kind == EPI_GATED_RES || e0.kind == EPI_RES_ADD) out = (double)(M0 + M1) * N * 8;
+  else if (e0.kind == EPI_QKV || e0.kind == EPI_GELU) out = (double)(M0 + M1) * N * es;
+  q.pre(BAG_PROF_GEMM, 2.0 * (M0 + M1) * N * K, ((double)M0 + M1 + 2.0 * N) * K * es + out,
+        M0 + M1, N, K);
+  q.chk(gemm2(A0, lda0, W0.p, ldw0, M0, e0, A1, lda1, W1.p, ldw1, M1, e1, N, K,
+              q.ctx->st ? &q.ctx->st->err : nullptr, q.s));
+}
+
 static void enq_ln(Enq& q, const float* x, long ldx, void* y, long ldy, int rows, int split,
                    const float* sh_a, const float* sc_a, const float* sh_b, const float* sc_b,
                    const DevState* st, int flag_want) {
@@ -690,11 +710,11 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw) {
       Epi e = base_epi(ctx, st, fw);
       enq_qkv_epi(ctx, e, nx, true);
       e.bias = (const float*)blk.w.at("img_qkv_b").p;
-      enq_gemm(q, off_act(ctx, ctx->xn, (long)nx * d), d, blk.w.at("img_qkv_w"), d, ni, (int)(3 * d), (int)d, e);
       Epi e2 = base_epi(ctx, st, fw);
       enq_qkv_epi(ctx, e2, 0, true);
       e2.bias = (const float*)blk.w.at("txt_qkv_b").p;
-      enq_gemm(q, ctx->xn, d, blk.w.at("txt_qkv_w"), d, nx, (int)(3 * d), (int)d, e2);
+      enq_gemm2(q, off_act(ctx, ctx->xn, (long)nx * d), d, blk.w.at("img_qkv_w"), d, ni, e,
+                ctx->xn, d, blk.w.at("txt_qkv_w"), d, nx, e2, (int)(3 * d), (int)d);
     }
     enq_attn(q, ctx->q, ctx->k, ctx->vt, ctx->vpad, ctx->cat, ldc, N, N, st, fw);
     {
@@ -705,12 +725,12 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw) {
       r.ldr = d;
       r.gate = mi + 2 * d;
       r.gate_step = ms;
-      enq_gemm(q, off_act(ctx, ctx->cat, (long)nx * ldc), ldc, blk.w.at("img_proj_w"), d, ni, (int)d, (int)d, r);
       Epi r2 = r;
       r2.bias = (const float*)blk.w.at("txt_proj_b").p;
       r2.resid = h;
       r2.gate = mt + 2 * d;
-      enq_gemm(q, ctx->cat, ldc, blk.w.at("txt_proj_w"), d, nx, (int)d, (int)d, r2);
+      enq_gemm2(q, off_act(ctx, ctx->cat, (long)nx * ldc), ldc, blk.w.at("img_proj_w"), d, ni, r,
+                ctx->cat, ldc, blk.w.at("txt_proj_w"), d, nx, r2, (int)d, (int)d);
     }
     // MLP half
     enq_ln(q, h, d, ctx->xn, d, N, nx, mt + 3 * d, mt + 4 * d, mi + 3 * d, mi + 4 * d, st, fw);
@@ -721,11 +741,11 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw) {
       u.ldo = ldc;
       u.bias = (const float*)blk.w.at("img_up_b").p;
       u.out = off_act(ctx, ctx->cat, (long)nx * ldc + d);
-      enq_gemm(q, off_act(ctx, ctx->xn, (long)nx * d), d, blk.w.at("img_up_w"), d, ni, (int)F, (int)d, u);
       Epi u2 = u;
       u2.bias = (const float*)blk.w.at("txt_up_b").p;
       u2.out = off_act(ctx, ctx->cat, d);
-      enq_gemm(q, ctx->xn, d, blk.w.at("txt_up_w"), d, nx, (int)F, (int)d, u2);
+      enq_gemm2(q, off_act(ctx, ctx->xn, (long)nx * d), d, blk.w.at("img_up_w"), d, ni, u,
+                ctx->xn, d, blk.w.at("txt_up_w"), d, nx, u2, (int)F, (int)d);
       Epi r = base_epi(ctx, st, fw);
       r.kind = EPI_GATED_RES;
       r.bias = (const float*)blk.w.at("img_down_b").p;
@@ -733,12 +753,12 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw) {
       r.ldr = d;
       r.gate = mi + 5 * d;
       r.gate_step = ms;
-      enq_gemm(q, off_act(ctx, ctx->cat, (long)nx * ldc + d), ldc, blk.w.at("img_down_w"), F, ni, (int)d, (int)F, r);
       Epi r2 = r;
       r2.bias = (const float*)blk.w.at("txt_down_b").p;
       r2.resid = h;
       r2.gate = mt + 5 * d;
-      enq_gemm(q, off_act(ctx, ctx->cat, d), ldc, blk.w.at("txt_down_w"), F, nx, (int)d, (int)F, r2);
+      enq_gemm2(q, off_act(ctx, ctx->cat, (long)nx * ldc + d), ldc, blk.w.at("img_down_w"), F, ni, r,
+                off_act(ctx, ctx->cat, d), ldc, blk.w.at("txt_down_w"), F, nx, r2, (int)d, (int)F);
     }
     return;
   }

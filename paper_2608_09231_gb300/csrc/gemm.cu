@@ -137,10 +137,15 @@ struct TcCfg {
 
 template <int BN>
 __global__ void __launch_bounds__(192, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const Epi e, int M, int N, int K, int a_split, int* err) {
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
+                   const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
+                   const __grid_constant__ Epi e0, const __grid_constant__ Epi e1, int M0, int M1,
+                   int N, int K, int a_split, int* err) {
+  // Two independent problems with the same N and K may share one launch (problem 1 has
+  // M1 rows, possibly 0): their tiles form one list, problem 0's first, so a small
+  // problem fills the SMs the large one leaves idle in its last wave.
   using C = TcCfg<BN>;
-  if (epi_skip(e.st, e.flag_want)) return;
+  if (epi_skip(e0.st, e0.flag_want)) return;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -155,12 +160,25 @@ __global__ void __launch_bounds__(192, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int num_m = (M + TC_BM - 1) / TC_BM, num_n = N / BN;
+  const int num_m0 = (M0 + TC_BM - 1) / TC_BM, num_m1 = (M1 + TC_BM - 1) / TC_BM, num_n = N / BN;
+  const int tiles0 = num_m0 * num_n;
+  auto decode = [&](int tile, int& pb, int& mt, int& nt) {
+    if (tile < tiles0) {
+      pb = 0;
+      mt = tile % num_m0;
+      nt = tile / num_m0;
+    } else {
+      const int l = tile - tiles0;
+      pb = 1;
+      mt = l % num_m1;
+      nt = l / num_m1;
+    }
+  };
   // a_split: A holds [hi | lo] bf16 halves of an fp32 activation ([M, 2K]); the K loop
   // runs twice as long, feeding each W chunk once with hi and once with lo, so the
   // product is accurate to fp32 accumulation while W is streamed once.
-  const int tiles = num_m * num_n, kit = (a_split ? 2 : 1) * (K / TC_BK);
-  const int t = epi_step(e);
+  const int tiles = tiles0 + num_m1 * num_n, kit = (a_split ? 2 : 1) * (K / TC_BK);
+  const int t = epi_step(e0);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
@@ -176,8 +194,12 @@ __global__ void __launch_bounds__(192, 1)
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&tmA);
-    tma_prefetch_desc(&tmB);
+    tma_prefetch_desc(&tmA0);
+    tma_prefetch_desc(&tmB0);
+    if (M1 > 0) {
+      tma_prefetch_desc(&tmA1);
+      tma_prefetch_desc(&tmB1);
+    }
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -196,7 +218,10 @@ __global__ void __launch_bounds__(192, 1)
       long issued = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
-        const int mt = tile % num_m, nt = tile / num_m;
+        int pb, mt, nt;
+        decode(tile, pb, mt, nt);
+        const CUtensorMap* tmA = pb ? &tmA1 : &tmA0;
+        const CUtensorMap* tmB = pb ? &tmB1 : &tmB0;
         for (int kb = 0; kb < kit; ++kb) {
           if (!mbar_wait(empty + s, ph ^ 1, abort_flag)) {
             ok = false;
@@ -205,8 +230,8 @@ __global__ void __launch_bounds__(192, 1)
           mbar_arrive_expect_tx(full + s, C::STAGE_BYTES);
           const int ka = a_split ? (kb & 1) * K + (kb >> 1) * TC_BK : kb * TC_BK;
           const int kw = a_split ? (kb >> 1) * TC_BK : kb * TC_BK;
-          tma_load_2d(sA + s * C::A_BYTES, &tmA, ka, mt * TC_BM, full + s);
-          tma_load_2d(sB + s * C::B_BYTES, &tmB, kw, nt * BN, full + s);
+          tma_load_2d(sA + s * C::A_BYTES, tmA, ka, mt * TC_BM, full + s);
+          tma_load_2d(sB + s * C::B_BYTES, tmB, kw, nt * BN, full + s);
           ++issued;
           if (++s == C::STAGES) {
             s = 0;
@@ -278,7 +303,9 @@ __global__ void __launch_bounds__(192, 1)
     int acc = 0;
     uint32_t aph = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
-      const int mt = tile % num_m, nt = tile / num_m;
+      int pb, mt, nt;
+      decode(tile, pb, mt, nt);
+      const Epi& e = pb ? e1 : e0;
       bool ok = mbar_wait(tfull + acc, aph, abort_flag);
       if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after();
@@ -305,16 +332,28 @@ __global__ void __launch_bounds__(192, 1)
 }
 
 template <int BN>
-static cudaError_t launch_tc(const void* A, long lda, const void* W, long ldw, int M, int N,
-                             int K, const Epi& e, int* err, cudaStream_t s, int a_split) {
+static cudaError_t launch_tc(const void* A0, long lda0, const void* W0, long ldw0, int M0,
+                             const Epi& e0, const void* A1, long lda1, const void* W1, long ldw1,
+                             int M1, const Epi& e1, int N, int K, int* err, cudaStream_t s,
+                             int a_split) {
   using C = TcCfg<BN>;
-  CUtensorMap ta, tb;
-  if (encode_tmap_2d_bf16(&ta, A, (uint64_t)K * (a_split ? 2 : 1), (uint64_t)M, (uint64_t)lda * 2, TC_BK, TC_BM) ||
-      encode_tmap_2d_bf16(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)ldw * 2, TC_BK, BN))
+  const uint64_t ka = (uint64_t)K * (a_split ? 2 : 1);
+  CUtensorMap ta0, tb0, ta1, tb1;
+  if (encode_tmap_2d_bf16(&ta0, A0, ka, (uint64_t)M0, (uint64_t)lda0 * 2, TC_BK, TC_BM) ||
+      encode_tmap_2d_bf16(&tb0, W0, (uint64_t)K, (uint64_t)N, (uint64_t)ldw0 * 2, TC_BK, BN))
     return cudaErrorInvalidValue;
-  const int tiles = ((M + TC_BM - 1) / TC_BM) * (N / BN);
+  if (M1 > 0) {
+    if (encode_tmap_2d_bf16(&ta1, A1, ka, (uint64_t)M1, (uint64_t)lda1 * 2, TC_BK, TC_BM) ||
+        encode_tmap_2d_bf16(&tb1, W1, (uint64_t)K, (uint64_t)N, (uint64_t)ldw1 * 2, TC_BK, BN))
+      return cudaErrorInvalidValue;
+  } else {
+    ta1 = ta0;
+    tb1 = tb0;
+  }
+  const int tiles = ((M0 + TC_BM - 1) / TC_BM + (M1 + TC_BM - 1) / TC_BM) * (N / BN);
   const int grid = std::min(tiles, num_sms());
-  gemm_tc_kernel<BN><<<grid, 192, C::SMEM, s>>>(ta, tb, e, M, N, K, a_split, err);
+  gemm_tc_kernel<BN><<<grid, 192, C::SMEM, s>>>(ta0, tb0, ta1, tb1, e0, e1, M0, M1, N, K,
+                                                a_split, err);
   return cudaGetLastError();
 }
 
@@ -340,6 +379,40 @@ int gemm_tc_supported(int M, int N, int K, long lda, long ldw) {
   return get_encode_fn() != nullptr;
 }
 
+// tensor-core launch of one or two problems (M1 = 0: one); picks the widest tile that
+// still gives every SM at least one tile
+static cudaError_t gemm_tc2(const void* A0, long lda0, const void* W0, long ldw0, int M0,
+                            const Epi& e0, const void* A1, long lda1, const void* W1, long ldw1,
+                            int M1, const Epi& e1, int N, int K, int* err, cudaStream_t s,
+                            int a_split) {
+  const uintptr_t ptrs = reinterpret_cast<uintptr_t>(A0) | reinterpret_cast<uintptr_t>(W0) |
+                         (M1 > 0 ? (reinterpret_cast<uintptr_t>(A1) | reinterpret_cast<uintptr_t>(W1)) : 0);
+  if ((ptrs & 15) || !gemm_tc_supported(M0, N, K, lda0, ldw0) ||
+      (M1 > 0 && !gemm_tc_supported(M1, N, K, lda1, ldw1)))
+    return cudaErrorNotSupported;
+  if (a_split && (lda0 < 2L * K || (M1 > 0 && lda1 < 2L * K))) return cudaErrorInvalidValue;
+  const int ns = num_sms();
+  const int mt = (M0 + TC_BM - 1) / TC_BM + (M1 + TC_BM - 1) / TC_BM;
+  if (N % 256 == 0 && mt * (N / 256) >= ns)
+    return launch_tc<256>(A0, lda0, W0, ldw0, M0, e0, A1, lda1, W1, ldw1, M1, e1, N, K, err, s, a_split);
+  if (N % 128 == 0 && mt * (N / 128) >= ns)
+    return launch_tc<128>(A0, lda0, W0, ldw0, M0, e0, A1, lda1, W1, ldw1, M1, e1, N, K, err, s, a_split);
+  return launch_tc<64>(A0, lda0, W0, ldw0, M0, e0, A1, lda1, W1, ldw1, M1, e1, N, K, err, s, a_split);
+}
+
+cudaError_t gemm2(const void* A0, long lda0, const void* W0, long ldw0, int M0, const Epi& epi0,
+                  const void* A1, long lda1, const void* W1, long ldw1, int M1, const Epi& epi1,
+                  int N, int K, int* err, cudaStream_t s) {
+  if (N <= 0 || (M0 <= 0 && M1 <= 0)) return cudaSuccess;
+  Epi e0 = epi0, e1 = epi1;
+  e0.M = M0;
+  e0.N = N;
+  e1.M = M1;
+  e1.N = N;
+  if (M0 <= 0) return gemm_tc2(A1, lda1, W1, ldw1, M1, e1, nullptr, 0, nullptr, 0, 0, e1, N, K, err, s, 0);
+  return gemm_tc2(A0, lda0, W0, ldw0, M0, e0, A1, lda1, W1, ldw1, M1 > 0 ? M1 : 0, e1, N, K, err, s, 0);
+}
+
 cudaError_t gemm(const void* A, long lda, const void* W, long ldw, int M, int N, int K,
                  int in_bf16, const Epi& epi_in, int* err, cudaStream_t s, int force_simt,
                  int a_split) {
@@ -347,17 +420,10 @@ cudaError_t gemm(const void* A, long lda, const void* W, long ldw, int M, int N,
   Epi e = epi_in;
   e.M = M;
   e.N = N;
-  const bool aligned = ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(W)) & 15) == 0;
   if (in_bf16 && !force_simt) {
     // bf16 operands always take the tensor-core path; a shape or pointer it cannot
     // tile is an error, never a silent switch to the CUDA-core kernel
-    if (!aligned || !gemm_tc_supported(M, N, K, lda, ldw)) return cudaErrorNotSupported;
-    if (a_split && lda < 2L * K) return cudaErrorInvalidValue;
-    const int ns = num_sms();
-    const int mt = (M + TC_BM - 1) / TC_BM;
-    if (N % 256 == 0 && mt * (N / 256) >= ns) return launch_tc<256>(A, lda, W, ldw, M, N, K, e, err, s, a_split);
-    if (N % 128 == 0 && mt * (N / 128) >= ns) return launch_tc<128>(A, lda, W, ldw, M, N, K, e, err, s, a_split);
-    return launch_tc<64>(A, lda, W, ldw, M, N, K, e, err, s, a_split);
+    return gemm_tc2(A, lda, W, ldw, M, e, nullptr, 0, nullptr, 0, 0, e, N, K, err, s, a_split);
   }
   if (a_split) return cudaErrorInvalidValue;
   if (N % 4 != 0) return cudaErrorInvalidValue;

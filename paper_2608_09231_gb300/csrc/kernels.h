@@ -95,6 +95,11 @@ cudaError_t gemm(const void* A, long lda, const void* W, long ldw, int M, int N,
 // dst [rows, 2*cols] bf16 = [bf16(x) | bf16(x - bf16(x))] of src fp32 [rows, cols]
 cudaError_t split_bf16(__nv_bfloat16* dst, const float* src, long rows, long cols, cudaStream_t s);
 int gemm_tc_supported(int M, int N, int K, long lda, long ldw);
+// Two bf16 problems with the same N and K in one tensor-core launch (e.g. the image and
+// text streams of a double-stream block); M1 may be 0.
+cudaError_t gemm2(const void* A0, long lda0, const void* W0, long ldw0, int M0, const Epi& epi0,
+                  const void* A1, long lda1, const void* W1, long ldw1, int M1, const Epi& epi1,
+                  int N, int K, int* err, cudaStream_t s);
 
 struct AttnArgs {
   const void* q;  long ldq;      // [Nq rows][ldq], head h at column h*dh
