@@ -102,39 +102,40 @@ class Clocks:
 # fp64 oracle on the host cores (CPU baseline and the reference arm)
 # ---------------------------------------------------------------------------
 def cpu_worker(cfg_name, reps, warm):
-    """Time the oracle's forward of one double-stream and one single-stream block at
-    full width and full token count; print per-rep seconds as JSON."""
+    """Time the oracle's forward of one block of each kind the stack has (double-stream,
+    single-stream, or Wan) at full width and full token count; print per-rep seconds."""
     import numpy as np
 
     from oracle import bag_oracle as O
     from paper_2608_09231_gb300 import configs, synth
 
     cfg = configs.get_config(cfg_name)
-    nd, ns = cfg["n_double"], cfg["n_single"]
-    pick = [0] + ([nd] if ns else [])
+    types = synth.block_types(cfg)
+    pick = sorted({types.index(t) for t in set(types)})
     W = O.to64(synth.make_weights(cfg, blocks=pick))
     G = W["global"]
     inp = synth.make_inputs(cfg)
-    d, H = cfg["hidden"], cfg["heads"]
+    H = cfg["heads"]
     vec = O.conditioning(cfg, G, 1.0, inp["pooled"].astype(np.float64))
     img = O.patch_embed(G, inp["x"].astype(np.float64))
     txt = inp["txt"].astype(np.float64)
     ang = O.rope_angles(O.token_positions(cfg), cfg["rope_axes"])
     out = []
     for r in range(warm + reps):
-        t0 = time.perf_counter()
-        blk = W["blocks"][0]
-        mod = O.block_modulation(cfg, G, blk, vec)
-        i2, t2 = O.double_block(img, txt, mod[0], mod[1], blk, ang, H)
-        t1 = time.perf_counter()
-        ts = 0.0
-        if ns:
-            blk = W["blocks"][nd]
-            hj = np.concatenate([t2, i2], axis=0)
-            O.single_block(hj, O.block_modulation(cfg, G, blk, vec), blk, ang, H)
-            ts = time.perf_counter() - t1
+        rec = {"double_s": 0.0, "single_s": 0.0, "wan_s": 0.0}
+        for b in pick:
+            blk = W["blocks"][b]
+            mod = O.block_modulation(cfg, G, blk, vec)
+            t0 = time.perf_counter()
+            if blk["type"] == "double":
+                O.double_block(img, txt, mod[0], mod[1], blk, ang, H)
+            elif blk["type"] == "single":
+                O.single_block(np.concatenate([txt, img], axis=0), mod, blk, ang, H)
+            else:
+                O.wan_block(img, txt, mod, blk, ang, H)
+            rec[blk["type"] + "_s"] = time.perf_counter() - t0
         if r >= warm:
-            out.append({"double_s": t1 - t0, "single_s": ts})
+            out.append(rec)
     print(json.dumps({"reps": out, "threads": os.cpu_count()}))
 
 
@@ -154,7 +155,8 @@ def run_cpu_oracle(cfg_name, reps, warm):
 
 def oracle_s_per_sample(cfg, B, rep):
     """Extrapolate one oracle sample: B full forwards of the whole stack."""
-    return B * (cfg["n_double"] * rep["double_s"] + cfg["n_single"] * rep["single_s"])
+    return B * (cfg["n_double"] * rep["double_s"] + cfg["n_single"] * rep["single_s"]
+                + cfg["n_wan"] * rep["wan_s"])
 
 
 # ---------------------------------------------------------------------------
@@ -359,8 +361,8 @@ def main():
                 "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config,
                 "cpu_baseline": {"value": v, "unit": "s/sample", "cores": res["threads"],
                                  "kind": "oracle",
-                                 "sample": "per step: one double-stream + one single-stream "
-                                           "block forward at full width and tokens, "
+                                 "sample": "per step: one block of each kind in the stack, "
+                                           "forward at full width and tokens in fp64, "
                                            "extrapolated linearly to B full stacks"},
                 "e2e": {"value": v, "unit": "s/sample", "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}}
@@ -500,9 +502,9 @@ def main():
             rep = res["reps"][0]
             cpu = {"value": oracle_s_per_sample(cfg, B, rep), "unit": "s/sample",
                    "cores": res["threads"], "kind": "oracle",
-                   "sample": (f"one double-stream block ({rep['double_s']:.1f} s) + one "
-                              f"single-stream block ({rep['single_s']:.1f} s) forward at full "
-                              f"width/tokens in fp64, extrapolated to B={B} full stacks")}
+                   "sample": ("one block of each kind at full width/tokens in fp64 ("
+                              + ", ".join(f"{k[:-2]} {v:.2f} s" for k, v in rep.items() if v)
+                              + f"), extrapolated to B={B} full stacks")}
         except Exception as ex:  # reported, never silently replaced
             cpu = {"value": None, "unit": "s/sample", "cores": os.cpu_count(), "kind": "oracle",
                    "sample": f"failed: {ex}"}
