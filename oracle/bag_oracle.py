@@ -362,6 +362,44 @@ def gate_logit(f, g):
     return z
 
 
+def gate_features6(B, T, c, t, t_last, drift, step):
+    """The six scalars of Eq. 3 in float32: s_bud = [B/T, (B-c)/B, (B-c)/(T-t)],
+    s_traj = [t - t_last, drift since the last full step, step-to-step change]."""
+    return [F32(B) / F32(T), F32(B - c) / F32(B), F32(B - c) / F32(T - t),
+            F32(t - t_last), F32(drift), F32(step)]
+
+
+def _dense32(x, W, b, relu):
+    """fp32 dense layer in a fixed order: out_j = b_j + sum_i W[j, i] x_i, inputs in index
+    order, every product and sum rounded on its own; optional ReLU."""
+    out = []
+    for j in range(W.shape[0]):
+        h = F32(b[j])
+        for i in range(len(x)):
+            h = F32(h + F32(F32(W[j, i]) * x[i]))
+        if relu and not h > F32(0.0):
+            h = F32(0.0)
+        out.append(h)
+    return out
+
+
+def gate_logit6(f, g):
+    """The paper's six-input gates (App. A.2) on z-scored inputs, fp32, ReLU hidden
+    activations: "flux6" one MLP 6-8-8-32-1; "wan6" budget branch 3-8-8 and trajectory
+    branch 3-8-8, concatenated [budget, trajectory], fused by 16-32-1."""
+    fz = [(F32(f[i]) - F32(g["mu"][i])) / F32(g["sd"][i]) for i in range(6)]
+    L = list(zip(g["W"], g["b"]))
+    if g["kind"] == "flux6":
+        h = fz
+        for k, (W, b) in enumerate(L):
+            h = _dense32(h, W, b, relu=k < len(L) - 1)
+        return h[0]
+    hb = _dense32(_dense32(fz[:3], *L[0], relu=True), *L[1], relu=True)
+    ht = _dense32(_dense32(fz[3:], *L[2], relu=True), *L[3], relu=True)
+    h = _dense32(hb + ht, *L[4], relu=True)
+    return _dense32(h, *L[5], relu=False)[0]
+
+
 def pace(gate_bit, B, T, c, t):
     """Algorithm 2's forced rules applied to the gate's bit at step t >= 1."""
     m = 1 if gate_bit else 0
@@ -397,7 +435,8 @@ def to64(W):
     return out
 
 
-def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=None):
+def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=None,
+           step_override=None):
     """One sample of T Euler steps under Algorithm 2.
 
     policy         'bag' (gate + pacing), 'full' (uncached: every step computes), or a
@@ -405,6 +444,8 @@ def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=Non
     drift_override optional per-step drift values (index t) to feed the gate instead of
                    the oracle's own; used to take the decision on another
                    implementation's logged gate inputs.
+    step_override  likewise for the step-to-step change (six-input gates).
+    The gate is the 3-input MLP unless gate["kind"] names a six-input gate.
     Returns dict(x=final latent, mask, log=[per-step dict]).
     """
     if not (1 <= B <= T):
@@ -434,8 +475,13 @@ def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=Non
             rec["s_bud"] = [B / T, (B - c) / B, (B - c) / (T - t)]
             rec["s_traj"] = [t - t_last, drift, rel_l1(m_t, m_prev)]
             used = drift if drift_override is None else drift_override[t]
-            f = gate_features(B, T, c, t, used)
-            z = gate_logit(f, gate)
+            if gate.get("kind", "mlp3") == "mlp3":
+                f = gate_features(B, T, c, t, used)
+                z = gate_logit(f, gate)
+            else:
+                step = rec["s_traj"][2] if step_override is None else step_override[t]
+                f = gate_features6(B, T, c, t, t_last, used, step)
+                z = gate_logit6(f, gate)
             rec["features"] = [float(v) for v in f]
             rec["z"] = float(z)
             gbit = 1 if z > thr else 0

@@ -263,8 +263,43 @@ def make_gate(gate_seed):
 
 
 def gate_flat(g):
-    """Flat parameter vector in the order w1 (row-major), b1, w2, b2 (81 floats)."""
-    return np.concatenate([g["w1"].ravel(), g["b1"], g["w2"], g["b2"]]).astype(np.float32)
+    """Flat parameter vector: for the 3-input gate w1 (row-major), b1, w2, b2 (81 floats);
+    for the 6-input gates every layer's W [out, in] (row-major) then b, in layer order."""
+    if g.get("kind", "mlp3") == "mlp3":
+        return np.concatenate([g["w1"].ravel(), g["b1"], g["w2"], g["b2"]]).astype(np.float32)
+    return np.concatenate([np.concatenate([W.ravel(), b]) for W, b in gate_layers(g)]).astype(np.float32)
+
+
+# The paper's six-input gates (App. A.2).  "flux6": one MLP 6 -> 8 -> 8 -> 32 -> 1 over
+# all six inputs; "wan6": a 3 -> 8 -> 8 branch on the budget inputs and one on the
+# trajectory inputs, concatenated and fused by 16 -> 32 -> 1.  Layer shapes as (out, in).
+GATE6_SHAPES = {
+    "flux6": [(8, 6), (8, 8), (32, 8), (1, 32)],
+    "wan6": [(8, 3), (8, 8), (8, 3), (8, 8), (32, 16), (1, 32)],
+}
+
+
+def gate_layers(g):
+    """The (W, b) pairs of a six-input gate in evaluation / storage order."""
+    return list(zip(g["W"], g["b"]))
+
+
+def make_gate6(gate_seed, kind):
+    """Seeded six-input gate: per layer W ~ U(-a, a) with a = sqrt(6 / (in + out)) and
+    b ~ U(-0.1, 0.1); tensor keys 1, 2, ... in storage order (W1, b1, W2, b2, ...)."""
+    Ws, bs = [], []
+    key = 1
+    for out, inn in GATE6_SHAPES[kind]:
+        a = float(np.sqrt(6.0 / (inn + out)))
+        Ws.append(uniform(gate_seed, key, out * inn, -a, a).reshape(out, inn))
+        bs.append(uniform(gate_seed, key + 1, out, -0.1, 0.1))
+        key += 2
+    return {"kind": kind, "W": Ws, "b": bs, "mu": np.zeros(6, np.float32),
+            "sd": np.ones(6, np.float32)}
+
+
+def make_gate_any(gate_seed, kind="mlp3"):
+    return make_gate(gate_seed) if kind == "mlp3" else make_gate6(gate_seed, kind)
 
 
 # Sample inputs: latent noise, text tokens and pooled vector, all N(0, 1).

@@ -544,3 +544,81 @@ def test_drift_is_zero_when_nothing_moves_and_logged_features():
         assert rec["s_traj"][0] == rec["t"] - max(
             q["t"] for q in r["log"][:rec["t"]] if q["full"])
         assert rec["features"][0] == np.float32(3 - rec["c_before"]) / np.float32(3)
+
+
+# ---------------------------------------------------------------------------
+# the paper's six-input gates (App. A.2) and the full state of Eq. 3
+# ---------------------------------------------------------------------------
+def test_six_input_gate_parameter_counts_match_the_paper():
+    with open(os.path.join(GOLDEN, "paper_values.json")) as f:
+        want = json.load(f)["gate_param_counts"]
+    assert synth.gate_flat(synth.make_gate6(5, "flux6")).size == want["flux"] == 449
+    assert synth.gate_flat(synth.make_gate6(5, "wan6")).size == want["wan"] == 785
+
+
+def test_six_features_closed_form():
+    f = O.gate_features6(B=20, T=50, c=5, t=10, t_last=7, drift=0.125, step=0.0625)
+    assert f == [np.float32(0.4), np.float32(0.75), np.float32(15) / np.float32(40),
+                 np.float32(3.0), np.float32(0.125), np.float32(0.0625)]
+
+
+def _relu(x):
+    return np.maximum(x, 0.0)
+
+
+@pytest.mark.parametrize("kind", ["flux6", "wan6"])
+def test_six_input_gate_matches_fp64_forward(kind):
+    """Fixed-order fp32 evaluation equals a float64 forward pass to rounding; the fp64
+    pass spells out the architecture (layer order; Wan: budget branch on inputs 0-2,
+    trajectory branch on 3-5, concatenated budget-first)."""
+    rng = np.random.default_rng(2)
+    for seed in range(10):
+        g = synth.make_gate6(seed, kind)
+        g["mu"] = (rng.normal(size=6) * 0.1).astype(np.float32)
+        g["sd"] = (1 + rng.random(6)).astype(np.float32)
+        f = [np.float32(v) for v in rng.random(6) * 2]
+        z = float(O.gate_logit6(f, g))
+        x = (np.array(f, np.float64) - g["mu"]) / g["sd"]
+        Ws = [w.astype(np.float64) for w in g["W"]]
+        bs = [b.astype(np.float64) for b in g["b"]]
+        if kind == "flux6":
+            h = x
+            for k in range(3):
+                h = _relu(Ws[k] @ h + bs[k])
+            z64 = float((Ws[3] @ h + bs[3])[0])
+        else:
+            hb = _relu(Ws[1] @ _relu(Ws[0] @ x[:3] + bs[0]) + bs[1])
+            ht = _relu(Ws[3] @ _relu(Ws[2] @ x[3:] + bs[2]) + bs[3])
+            z64 = float((Ws[5] @ _relu(Ws[4] @ np.r_[hb, ht] + bs[4]) + bs[5])[0])
+        assert abs(z - z64) <= 1e-5 * (1 + abs(z64))
+
+
+def test_wan_gate_branches_read_their_own_inputs():
+    """With only the trajectory branch's path to the output open and identity-like
+    weights, z = relu(t - t_last) - 2: the branch reads input 3 (staleness)."""
+    g = synth.make_gate6(1, "wan6")
+    for W in g["W"]:
+        W[:] = 0.0
+    for b in g["b"]:
+        b[:] = 0.0
+    g["W"][2][0, 0] = 1.0      # trajectory branch layer 1: input 0 of its slice = t - t_last
+    g["W"][3][0, 0] = 1.0      # trajectory branch layer 2
+    g["W"][4][0, 8] = 1.0      # fuse layer reads the first trajectory feature (index 8)
+    g["W"][5][0, 0] = 1.0
+    g["b"][5][0] = -2.0
+    f = O.gate_features6(B=20, T=50, c=5, t=10, t_last=7, drift=0.5, step=0.5)
+    assert O.gate_logit6(f, g) == np.float32(1.0)
+    f = O.gate_features6(B=20, T=50, c=5, t=10, t_last=9, drift=0.5, step=0.5)
+    assert O.gate_logit6(f, g) == np.float32(-1.0)
+
+
+@pytest.mark.parametrize("kind", ["flux6", "wan6"])
+def test_six_input_gates_spend_exactly_B(kind):
+    cfg, W, _, inp = _tiny(grid=(1, 4, 4), n_txt=3)
+    g = synth.make_gate6(cfg["gate_seed"], kind)
+    for B in (1, 4, 7):
+        r = O.sample(cfg, W, g, inp, T=7, B=B)
+        assert r["nfe"] == B and r["mask"][0] == 1
+        for rec in r["log"][1:]:
+            assert len(rec["features"]) == 6
+            assert rec["features"][3] == rec["s_traj"][0]
