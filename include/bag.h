@@ -42,6 +42,13 @@ typedef enum {
 
 enum { BAG_KIND_SINGLE = 0, BAG_KIND_MMDIT = 1, BAG_KIND_WAN = 2 };
 enum { BAG_F32 = 0, BAG_BF16 = 1 };
+/* Gate architectures (Eq. 1; the six-input ones are App. A.2's).  MLP3: inputs
+ * [(B-c)/B, (T-t)/T, drift], 3 -> 16 -> 1 (81 params).  FLUX6: the six scalars of Eq. 3
+ * [B/T, (B-c)/B, (B-c)/(T-t), t - t_last, drift, step change], 6 -> 8 -> 8 -> 32 -> 1
+ * (449 params).  WAN6: the same six inputs, budget (first three) and trajectory (last
+ * three) branches 3 -> 8 -> 8 each, concatenated budget-first, 16 -> 32 -> 1 (785
+ * params).  Hidden layers use ReLU; the decision is sigmoid(z) > tau. */
+enum { BAG_GATE_MLP3 = 0, BAG_GATE_FLUX6 = 1, BAG_GATE_WAN6 = 2 };
 enum {
   BAG_POLICY_BAG = 0,   /* Algorithm 2: gate decision + the two forced pacing rules */
   BAG_POLICY_FULL = 1,  /* uncached sampling: every step evaluates the network */
@@ -66,6 +73,7 @@ typedef struct {
   int dtype;          /* BAG_F32 or BAG_BF16 */
   uint64_t weight_seed, gate_seed;
   float tau;          /* gate cutoff: a step computes when sigmoid(z) > tau (0 < tau < 1) */
+  int gate_kind;      /* BAG_GATE_* */
 } bag_arch;
 
 /* Conditioning of one sample (device pointers, read during bag_step / bag_run).
@@ -79,9 +87,10 @@ typedef struct {
 
 /* Per-sample schedule statistics.  mask / log are optional host arrays supplied by the
  * caller: mask[T] receives m_t, log[T * BAG_LOG_FLOATS] the per-step record
- *   [0..2] gate inputs (B-c)/B, (T-t)/T, drift;  [3] gate logit z;  [4] raw gate bit;
- *   [5] m_t;  [6] c before the step;  [7] t - t_last;  [8..10] B/T, (B-c)/B,
- *   (B-c)/(T-t);  [11] sum|m_t - m_last|;  [12] sum|m_last|.
+ *   [0..2] (B-c)/B, (T-t)/T, drift;  [3] gate logit z;  [4] raw gate bit;  [5] m_t;
+ *   [6] c before the step;  [7] t - t_last;  [8..10] B/T, (B-c)/B, (B-c)/(T-t);
+ *   [11] sum|m_t - m_last|;  [12] sum|m_last|;  [13] step change;  [14] sum|m_t - m_{t-1}|;
+ *   [15] sum|m_{t-1}|   (m = the first block's modulated image-stream input).
  * nfe receives the realised number of full evaluations. */
 #define BAG_LOG_FLOATS 16
 typedef struct {
@@ -114,9 +123,12 @@ const char* bag_last_error(bag_ctx* ctx);
 bag_status bag_set_stream(bag_ctx* ctx, void* cuda_stream);
 
 /* Replace the gate parameters (Eq. 1; App. A.2 z-scored inputs).  theta: host array of
- * 81 floats = W1[16][3] row-major, b1[16], w2[16], b2; mu, sd: host arrays of 3 floats
- * (z-score statistics; null = 0 and 1). */
-bag_status bag_load_gate(bag_ctx* ctx, const float* theta, const float* mu, const float* sd);
+ * n floats, every layer's W [out][in] (row-major) then its b, in the order listed with
+ * BAG_GATE_* (WAN6: budget branch, trajectory branch, fuse layers); n must equal the
+ * kind's parameter count (81, 449 or 785) else EINVAL.  mu, sd: host arrays with one
+ * float per gate input (3 or 6; z-score statistics; null = 0 and 1; sd nonzero). */
+bag_status bag_load_gate(bag_ctx* ctx, const float* theta, int n, const float* mu,
+                         const float* sd);
 
 /* Choose the schedule policy (BAG_POLICY_*).  For BAG_POLICY_MASK, host_mask[T] gives
  * the per-step bits (host_mask[0] is ignored: step 0 always computes).  The budget

@@ -18,6 +18,7 @@ LIB_PATH = os.path.join(_HERE, "libbag.so")
 
 KIND = {"single": 0, "mmdit": 1, "wan": 2}
 DTYPE = {"f32": 0, "bf16": 1}
+GATE_KIND = {"mlp3": 0, "flux6": 1, "wan6": 2}
 POLICY_BAG, POLICY_FULL, POLICY_MASK = 0, 1, 2
 LOG_FLOATS = 16
 STATUS = {0: "BAG_OK", 1: "BAG_EINVAL", 2: "BAG_ENOMEM", 3: "BAG_ECUDA", 4: "BAG_EORDER",
@@ -44,7 +45,8 @@ class Arch(ctypes.Structure):
                 ("n_wan", ctypes.c_int), ("grid", ctypes.c_int * 3), ("n_txt", ctypes.c_int),
                 ("patch_ch", ctypes.c_int), ("rope_axes", ctypes.c_int * 3),
                 ("dtype", ctypes.c_int), ("weight_seed", ctypes.c_uint64),
-                ("gate_seed", ctypes.c_uint64), ("tau", ctypes.c_float)]
+                ("gate_seed", ctypes.c_uint64), ("tau", ctypes.c_float),
+                ("gate_kind", ctypes.c_int)]
 
 
 class Cond(ctypes.Structure):
@@ -88,7 +90,7 @@ def load(path=None):
         "bag_destroy": ([_P], None),
         "bag_last_error": ([_P], ctypes.c_char_p),
         "bag_set_stream": ([_P, _P], _I),
-        "bag_load_gate": ([_P, _P, _P, _P], _I),
+        "bag_load_gate": ([_P, _P, _I, _P, _P], _I),
         "bag_set_policy": ([_P, _I, _P], _I),
         "bag_reset": ([_P], _I),
         "bag_step": ([_P, _P, _I, ctypes.POINTER(Cond), _P, _P], _I),
@@ -127,6 +129,7 @@ def arch_from_config(cfg, tau=0.5):
     a.dtype = DTYPE[cfg["dtype"]]
     a.weight_seed, a.gate_seed = cfg["weight_seed"], cfg["gate_seed"]
     a.tau = tau
+    a.gate_kind = GATE_KIND[cfg.get("gate_kind", "mlp3")]
     return a
 
 
@@ -172,7 +175,7 @@ class Context:
         th = np.ascontiguousarray(theta, np.float32)
         mu_a = None if mu is None else np.ascontiguousarray(mu, np.float32)
         sd_a = None if sd is None else np.ascontiguousarray(sd, np.float32)
-        self._chk(self.lib.bag_load_gate(self.h, th.ctypes.data,
+        self._chk(self.lib.bag_load_gate(self.h, th.ctypes.data, th.size,
                                          None if mu_a is None else mu_a.ctypes.data,
                                          None if sd_a is None else sd_a.ctypes.data))
 

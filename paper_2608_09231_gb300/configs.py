@@ -24,6 +24,7 @@ n_txt       text tokens (joint attention) or context tokens (Wan cross-attention
 patch_ch    channels per image token in the latent (64 = 16-ch latent x 2x2 patch)
 rope_axes   head-dim split of the rotary embedding over the (frame, row, col) axes
 dtype       'f32' or 'bf16' (GEMM / attention operand type)
+gate_kind   'mlp3' (3 inputs, default), 'flux6' or 'wan6' (the paper's six-input gates)
 """
 
 import copy
@@ -80,6 +81,7 @@ def get_config(name, **overrides):
     else:
         raise KeyError(f"unknown config {name!r}")
     cfg.update(overrides)
+    cfg.setdefault("gate_kind", "mlp3")
     cfg["name"] = name
     d, h = cfg["hidden"], cfg["heads"]
     assert d % h == 0

@@ -84,7 +84,6 @@ const std::map<std::string, int> kWanIds = {
     {"ffn_up_w", 11}, {"ffn_up_b", 12}, {"ffn_down_w", 13}, {"ffn_down_b", 14}};
 
 constexpr int kTembDim = 256;
-constexpr int kGateFloats = 87;
 
 }  // namespace
 
@@ -230,6 +229,7 @@ static bag_status validate_arch(const bag_arch* a, int T, int B) {
   if (a->kind == BAG_KIND_SINGLE && a->n_double) return fail(nullptr, BAG_EINVAL, "SINGLE kind has no double blocks");
   if (!(a->tau > 0.f && a->tau < 1.f)) return fail(nullptr, BAG_EINVAL, "tau must be in (0, 1)");
   if (a->dtype != BAG_F32 && a->dtype != BAG_BF16) return fail(nullptr, BAG_EINVAL, "dtype");
+  if (a->gate_kind < BAG_GATE_MLP3 || a->gate_kind > BAG_GATE_WAN6) return fail(nullptr, BAG_EINVAL, "gate_kind");
   return BAG_OK;
 }
 
@@ -415,19 +415,37 @@ static bag_status seed_weights(bag_ctx* ctx) {
   return BAG_OK;
 }
 
+// Layer shapes (out, in) of each gate kind, in evaluation / storage order (Eq. 1; the
+// six-input architectures are App. A.2's: 449 and 785 parameters).
+static std::vector<std::pair<int, int>> gate_shapes(int kind) {
+  if (kind == BAG_GATE_FLUX6) return {{8, 6}, {8, 8}, {32, 8}, {1, 32}};
+  if (kind == BAG_GATE_WAN6) return {{8, 3}, {8, 8}, {8, 3}, {8, 8}, {32, 16}, {1, 32}};
+  return {{16, 3}, {1, 16}};
+}
+static int gate_param_count(int kind) {
+  int n = 0;
+  for (auto& s : gate_shapes(kind)) n += s.first * s.second + s.first;
+  return n;
+}
+static int gate_inputs(int kind) { return kind == BAG_GATE_MLP3 ? 3 : 6; }
+
 static bag_status seed_gate(bag_ctx* ctx) {
-  float g[kGateFloats];
+  // per layer W ~ U(-a, a), a = sqrt(6 / (in + out)) and b ~ U(-0.1, 0.1); generator keys
+  // 1, 2, ... in storage order; z-score statistics 0 and 1
+  std::vector<float> g(kGateFloats, 0.f);
   const uint64_t s = ctx->arch.gate_seed;
-  const double a1 = std::sqrt(6.0 / 19.0), a2 = std::sqrt(6.0 / 17.0);
-  sm_uniform(s, 1, 48, -a1, a1, g);
-  sm_uniform(s, 2, 16, -0.1, 0.1, g + 48);
-  sm_uniform(s, 3, 16, -a2, a2, g + 64);
-  sm_uniform(s, 4, 1, -0.1, 0.1, g + 80);
-  for (int i = 0; i < 3; ++i) {
-    g[81 + i] = 0.f;
-    g[84 + i] = 1.f;
+  uint64_t key = 1;
+  int off = 0;
+  for (auto& sh : gate_shapes(ctx->arch.gate_kind)) {
+    const double a = std::sqrt(6.0 / (sh.first + sh.second));
+    sm_uniform(s, key, sh.first * sh.second, -a, a, g.data() + off);
+    off += sh.first * sh.second;
+    sm_uniform(s, key + 1, sh.first, -0.1, 0.1, g.data() + off);
+    off += sh.first;
+    key += 2;
   }
-  CK(cudaMemcpy(ctx->d_gate, g, sizeof(g), cudaMemcpyHostToDevice));
+  for (int i = 0; i < 6; ++i) g[kGateSd + i] = 1.f;
+  CK(cudaMemcpy(ctx->d_gate, g.data(), g.size() * 4, cudaMemcpyHostToDevice));
   return BAG_OK;
 }
 
@@ -473,7 +491,7 @@ static bag_status alloc_activations(bag_ctx* ctx) {
   A.add((void**)&ctx->R, (size_t)ni * d * 4);
   A.add(&ctx->m_cur, (size_t)ni * d * es);
   A.add(&ctx->m_last, (size_t)ni * d * es);
-  A.add((void**)&ctx->sig_partial, (size_t)ni * 2 * 4);
+  A.add((void**)&ctx->sig_partial, (size_t)ni * 4 * 4);
   A.add(&ctx->xn, (size_t)rows * d * es);
   A.add(&ctx->q, (size_t)rows * d * es);
   A.add(&ctx->k, (size_t)rows * d * es);
@@ -867,6 +885,7 @@ static void enq_prefix(Enq& q, int use_cond, unsigned long long handle) {
   a.scale_a = a.scale_b = m0 + d;
   a.mod_step = ctx->mod_stride;
   a.sig_ref = ctx->m_last;
+  a.sig_ref2 = ctx->m_cur;  // still the previous step's observable; replaced in place
   a.sig_partial = ctx->sig_partial;
   a.sig_on = 1;
   a.st = ctx->st;
@@ -874,7 +893,7 @@ static void enq_prefix(Enq& q, int use_cond, unsigned long long handle) {
   q.pre(BAG_PROF_SIGNAL, 0.0, (double)ctx->ni * d * (4.0 + 2.0 * ctx->act_size));
   q.chk(ln_mod(a, q.s));
   q.pre(BAG_PROF_GATE, 0.0, (double)ctx->ni * 8);
-  q.chk(gate_step(ctx->st, ctx->sig_partial, ctx->ni, ctx->d_gate, ctx->thr, ctx->T, ctx->B,
+  q.chk(gate_step(ctx->st, ctx->sig_partial, ctx->ni, ctx->d_gate, ctx->arch.gate_kind, ctx->thr, ctx->T, ctx->B,
                   ctx->policy, ctx->d_pmask, ctx->log, handle, use_cond, q.s));
 }
 
@@ -1430,17 +1449,23 @@ bag_status bag_set_stream(bag_ctx* ctx, void* stream) {
   return BAG_OK;
 }
 
-bag_status bag_load_gate(bag_ctx* ctx, const float* theta, const float* mu, const float* sd) {
+bag_status bag_load_gate(bag_ctx* ctx, const float* theta, int n, const float* mu, const float* sd) {
   if (!ctx) return BAG_EINVAL;
   if (!theta) return fail(ctx, BAG_EINVAL, "theta is null");
-  float g[kGateFloats];
-  std::memcpy(g, theta, 81 * sizeof(float));
-  for (int i = 0; i < 3; ++i) {
-    g[81 + i] = mu ? mu[i] : 0.f;
-    g[84 + i] = sd ? sd[i] : 1.f;
-    if (!(g[84 + i] != 0.f)) return fail(ctx, BAG_EINVAL, "sd must be nonzero");
+  const int kind = ctx->arch.gate_kind;
+  if (n != gate_param_count(kind))
+    return fail(ctx, BAG_EINVAL, "gate kind " + std::to_string(kind) + " has " +
+                                     std::to_string(gate_param_count(kind)) + " parameters, got " +
+                                     std::to_string(n));
+  std::vector<float> g(kGateFloats, 0.f);
+  std::memcpy(g.data(), theta, (size_t)n * sizeof(float));
+  for (int i = 0; i < 6; ++i) g[kGateSd + i] = 1.f;
+  for (int i = 0; i < gate_inputs(kind); ++i) {
+    g[kGateMu + i] = mu ? mu[i] : 0.f;
+    g[kGateSd + i] = sd ? sd[i] : 1.f;
+    if (!(g[kGateSd + i] != 0.f)) return fail(ctx, BAG_EINVAL, "sd must be nonzero");
   }
-  CK(cudaMemcpyAsync(ctx->d_gate, g, sizeof(g), cudaMemcpyHostToDevice, ctx->stream));
+  CK(cudaMemcpyAsync(ctx->d_gate, g.data(), g.size() * 4, cudaMemcpyHostToDevice, ctx->stream));
   CK(cudaStreamSynchronize(ctx->stream));
   return BAG_OK;
 }

@@ -37,6 +37,24 @@ BAG_DEV float block_sum(float v, float* red) {
   return s;
 }
 
+BAG_DEV void load4(const void* p, long off, int bf16, float* r) {
+  if (bf16) {
+    const uint2 u = *reinterpret_cast<const uint2*>(reinterpret_cast<const __nv_bfloat16*>(p) + off);
+    const __nv_bfloat162 r01 = *reinterpret_cast<const __nv_bfloat162*>(&u.x);
+    const __nv_bfloat162 r23 = *reinterpret_cast<const __nv_bfloat162*>(&u.y);
+    r[0] = __low2float(r01);
+    r[1] = __high2float(r01);
+    r[2] = __low2float(r23);
+    r[3] = __high2float(r23);
+  } else {
+    const float4 r4 = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(p) + off);
+    r[0] = r4.x;
+    r[1] = r4.y;
+    r[2] = r4.z;
+    r[3] = r4.w;
+  }
+}
+
 __global__ void __launch_bounds__(LN_THREADS) ln_mod_kernel(const LnArgs a) {
   if (epi_skip(a.st, a.flag_want)) return;
   __shared__ float red[LN_THREADS / 32];
@@ -71,7 +89,7 @@ __global__ void __launch_bounds__(LN_THREADS) ln_mod_kernel(const LnArgs a) {
   const float* sc = first ? a.scale_a : a.scale_b;
   if (sh) sh += (long)t * a.mod_step;
   if (sc) sc += (long)t * a.mod_step;
-  float sig_num = 0.f, sig_den = 0.f;
+  float sig_num = 0.f, sig_den = 0.f, sig_num2 = 0.f, sig_den2 = 0.f;
 #pragma unroll
   for (int i = 0; i < LN_MAXV; ++i) {
     const int c = threadIdx.x + i * LN_THREADS;
@@ -93,6 +111,21 @@ __global__ void __launch_bounds__(LN_THREADS) ln_mod_kernel(const LnArgs a) {
         y[3] += h4.w;
       }
       const long off = (long)row * a.ldy + 4 * c;
+      if (a.sig_on) {
+        // both references are read before y is stored: sig_ref2 may be the y buffer
+        // itself (the previous step's observable, replaced by this step's)
+        float r[4], r2[4], yy[4];
+        load4(a.sig_ref, off, a.y_bf16, r);
+        load4(a.sig_ref2, off, a.y_bf16, r2);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          yy[j] = a.y_bf16 ? bf16_round(y[j]) : y[j];
+          sig_num += fabsf(yy[j] - r[j]);
+          sig_den += fabsf(r[j]);
+          sig_num2 += fabsf(yy[j] - r2[j]);
+          sig_den2 += fabsf(r2[j]);
+        }
+      }
       if (a.y_bf16) {
         uint2 u;
         u.x = pack_bf16x2(y[0], y[1]);
@@ -102,43 +135,18 @@ __global__ void __launch_bounds__(LN_THREADS) ln_mod_kernel(const LnArgs a) {
         *reinterpret_cast<float4*>(reinterpret_cast<float*>(a.y) + off) =
             make_float4(y[0], y[1], y[2], y[3]);
       }
-      if (a.sig_on) {
-        float r[4], yy[4];
-        if (a.y_bf16) {
-          const uint2 u = *reinterpret_cast<const uint2*>(
-              reinterpret_cast<const __nv_bfloat16*>(a.sig_ref) + off);
-          const __nv_bfloat162 r01 = *reinterpret_cast<const __nv_bfloat162*>(&u.x);
-          const __nv_bfloat162 r23 = *reinterpret_cast<const __nv_bfloat162*>(&u.y);
-          r[0] = __low2float(r01);
-          r[1] = __high2float(r01);
-          r[2] = __low2float(r23);
-          r[3] = __high2float(r23);
-#pragma unroll
-          for (int j = 0; j < 4; ++j) yy[j] = bf16_round(y[j]);
-        } else {
-          const float4 r4 = *reinterpret_cast<const float4*>(
-              reinterpret_cast<const float*>(a.sig_ref) + off);
-          r[0] = r4.x;
-          r[1] = r4.y;
-          r[2] = r4.z;
-          r[3] = r4.w;
-#pragma unroll
-          for (int j = 0; j < 4; ++j) yy[j] = y[j];
-        }
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          sig_num += fabsf(yy[j] - r[j]);
-          sig_den += fabsf(r[j]);
-        }
-      }
     }
   }
   if (a.sig_on) {
     const float n = block_sum(sig_num, red);
     const float d = block_sum(sig_den, red);
+    const float n2 = block_sum(sig_num2, red);
+    const float d2 = block_sum(sig_den2, red);
     if (threadIdx.x == 0) {
-      a.sig_partial[2 * row] = n;
-      a.sig_partial[2 * row + 1] = d;
+      a.sig_partial[4 * row] = n;
+      a.sig_partial[4 * row + 1] = d;
+      a.sig_partial[4 * row + 2] = n2;
+      a.sig_partial[4 * row + 3] = d2;
     }
   }
 }
@@ -213,44 +221,87 @@ cudaError_t rel_l1_finalize(const float* partial, long rows, float* out, cudaStr
 // ---------------------------------------------------------------------------
 // gate + pacing (one warp)
 // ---------------------------------------------------------------------------
-// gate_params layout: w1[16][3] (row-major), b1[16], w2[16], b2, mu[3], sd[3]
+// Gate parameters: every layer's W [out][in] (row-major) then b, in evaluation order,
+// from offset 0; z-score mean at kGateMu, standard deviation at kGateSd (3 or 6 used).
+//   kind 0 (3 inputs): 3 -> 16 -> 1
+//   kind 1 (6 inputs): 6 -> 8 -> 8 -> 32 -> 1
+//   kind 2 (6 inputs): [budget 3 -> 8 -> 8 | trajectory 3 -> 8 -> 8] -> 16 -> 32 -> 1
+// Every hidden layer is followed by ReLU.  Each dense layer runs in a fixed order (bias
+// first, then inputs in index order, every product and sum rounded on its own) so the
+// logit is reproducible bit for bit by any IEEE fp32 evaluation in the same order.
+BAG_DEV const float* dense32(const float* p, int out, int in, const float* x, float* y, bool relu) {
+  const float* W = p;
+  const float* b = p + out * in;
+  for (int j = 0; j < out; ++j) {
+    float h = b[j];
+    for (int i = 0; i < in; ++i) h = __fadd_rn(h, __fmul_rn(W[j * in + i], x[i]));
+    if (relu && !(h > 0.f)) h = 0.f;
+    y[j] = h;
+  }
+  return b + out;
+}
+
 __global__ void gate_kernel(DevState* st, const float* partial, int rows, const float* gp,
-                            float thr, int T, int B, int policy, const uint8_t* pmask, float* log,
-                            cudaGraphConditionalHandle handle, int use_cond) {
+                            int kind, float thr, int T, int B, int policy, const uint8_t* pmask,
+                            float* log, cudaGraphConditionalHandle handle, int use_cond) {
   const int lane = threadIdx.x;
   const int t = st->t, c = st->c, t_last = st->t_last;
-  float num = 0.f, den = 0.f;
+  float num = 0.f, den = 0.f, num2 = 0.f, den2 = 0.f;
   if (t > 0) {
     for (int r = lane; r < rows; r += 32) {
-      num += partial[2 * r];
-      den += partial[2 * r + 1];
+      num += partial[4 * r];
+      den += partial[4 * r + 1];
+      num2 += partial[4 * r + 2];
+      den2 += partial[4 * r + 3];
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
       num += __shfl_xor_sync(0xffffffffu, num, off);
       den += __shfl_xor_sync(0xffffffffu, den, off);
+      num2 += __shfl_xor_sync(0xffffffffu, num2, off);
+      den2 += __shfl_xor_sync(0xffffffffu, den2, off);
     }
   }
   if (lane != 0) return;
   float* L = log + (long)t * kLogFloats;
   int m = 1, gbit = 1;
-  float z = 0.f, f0 = 0.f, f1 = 0.f, f2 = 0.f;
+  float z = 0.f, f0 = 0.f, f1 = 0.f, drift = 0.f, step = 0.f;
+  float sb[3] = {0.f, 0.f, 0.f};
   if (t > 0) {
     f0 = __fdiv_rn((float)(B - c), (float)B);
     f1 = __fdiv_rn((float)(T - t), (float)T);
-    f2 = __fdiv_rn(num, den);
-    const float f[3] = {f0, f1, f2};
-    float fz[3];
-#pragma unroll
-    for (int i = 0; i < 3; ++i) fz[i] = __fdiv_rn(__fsub_rn(f[i], gp[81 + i]), gp[84 + i]);
-    z = gp[80];
-    for (int j = 0; j < 16; ++j) {
-      float h = gp[48 + j];
-#pragma unroll
-      for (int i = 0; i < 3; ++i) h = __fadd_rn(h, __fmul_rn(gp[3 * j + i], fz[i]));
-      if (!(h > 0.f)) h = 0.f;
-      z = __fadd_rn(z, __fmul_rn(gp[64 + j], h));
+    drift = __fdiv_rn(num, den);
+    step = __fdiv_rn(num2, den2);
+    sb[0] = __fdiv_rn((float)B, (float)T);
+    sb[1] = f0;
+    sb[2] = __fdiv_rn((float)(B - c), (float)(T - t));
+    const float* mu = gp + kGateMu;
+    const float* sd = gp + kGateSd;
+    float x[6], h1[32], h2[32];
+    if (kind == 0) {
+      const float f[3] = {f0, f1, drift};
+      for (int i = 0; i < 3; ++i) x[i] = __fdiv_rn(__fsub_rn(f[i], mu[i]), sd[i]);
+      const float* p = dense32(gp, 16, 3, x, h1, true);
+      dense32(p, 1, 16, h1, h2, false);
+    } else {
+      const float f[6] = {sb[0], sb[1], sb[2], (float)(t - t_last), drift, step};
+      for (int i = 0; i < 6; ++i) x[i] = __fdiv_rn(__fsub_rn(f[i], mu[i]), sd[i]);
+      if (kind == 1) {
+        const float* p = dense32(gp, 8, 6, x, h1, true);
+        p = dense32(p, 8, 8, h1, h2, true);
+        p = dense32(p, 32, 8, h2, h1, true);
+        dense32(p, 1, 32, h1, h2, false);
+      } else {
+        float hb[8], cat[16];
+        const float* p = dense32(gp, 8, 3, x, hb, true);
+        p = dense32(p, 8, 8, hb, cat, true);
+        p = dense32(p, 8, 3, x + 3, hb, true);
+        p = dense32(p, 8, 8, hb, cat + 8, true);
+        p = dense32(p, 32, 16, cat, h1, true);
+        dense32(p, 1, 32, h1, h2, false);
+      }
     }
+    z = h2[0];
     gbit = z > thr ? 1 : 0;
     if (policy == 0) {  // Algorithm 2
       m = gbit;
@@ -264,17 +315,20 @@ __global__ void gate_kernel(DevState* st, const float* partial, int rows, const 
   }
   L[0] = f0;
   L[1] = f1;
-  L[2] = f2;
+  L[2] = drift;
   L[3] = z;
   L[4] = (float)gbit;
   L[5] = (float)m;
   L[6] = (float)c;
   L[7] = t > 0 ? (float)(t - t_last) : 0.f;
-  L[8] = (float)B / (float)T;
-  L[9] = (float)(B - c) / (float)B;
-  L[10] = (float)(B - c) / (float)(T - t);
+  L[8] = sb[0];
+  L[9] = sb[1];
+  L[10] = sb[2];
   L[11] = num;
   L[12] = den;
+  L[13] = step;
+  L[14] = num2;
+  L[15] = den2;
   st->flag = m;
   if (m) {
     st->c = c + 1;
@@ -284,9 +338,9 @@ __global__ void gate_kernel(DevState* st, const float* partial, int rows, const 
 }
 
 cudaError_t gate_step(DevState* st, const float* sig_partial, int sig_rows, const float* gate_params,
-                      float thr, int T, int B, int policy, const uint8_t* policy_mask, float* log,
-                      unsigned long long cond_handle, int use_cond, cudaStream_t s) {
-  gate_kernel<<<1, 32, 0, s>>>(st, sig_partial, sig_rows, gate_params, thr, T, B, policy,
+                      int gate_kind, float thr, int T, int B, int policy, const uint8_t* policy_mask,
+                      float* log, unsigned long long cond_handle, int use_cond, cudaStream_t s) {
+  gate_kernel<<<1, 32, 0, s>>>(st, sig_partial, sig_rows, gate_params, gate_kind, thr, T, B, policy,
                                policy_mask, log, (cudaGraphConditionalHandle)cond_handle, use_cond);
   return cudaGetLastError();
 }

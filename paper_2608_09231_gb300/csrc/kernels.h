@@ -26,7 +26,13 @@ constexpr int kLogFloats = 16;
 // [4]     raw gate bit, [5] final decision m_t, [6] c before the step, [7] t - t_last
 // [8..10] budget state of Eq. 3: B/T, (B-c)/B, (B-c)/(T-t)
 // [11]    drift numerator sum|m_t - m_last|, [12] denominator sum|m_last|
-// [13..15] reserved
+// [13]    step-to-step change, [14] its numerator sum|m_t - m_{t-1}|, [15] sum|m_{t-1}|
+
+// gate parameter buffer: layers from 0, z-score mean / sd at fixed offsets
+constexpr int kGateMaxParams = 800;
+constexpr int kGateMu = 800;
+constexpr int kGateSd = 806;
+constexpr int kGateFloats = 812;
 
 enum EpiKind : int {
   EPI_STORE = 0,      // out = acc + bias                       (out_bf16 selects type)
@@ -123,16 +129,17 @@ struct LnArgs {
   const float* shift_a; const float* scale_a;
   const float* shift_b; const float* scale_b;
   long mod_step;
-  // fused trajectory signal: per-row partial sums of |y - ref| and |ref|; y also
-  // stored to sig_out (the reference for the next full step is copied from it).
-  const void* sig_ref; float* sig_partial; int sig_on;
+  // fused trajectory signal: per-row partial sums of |y - ref|, |ref|, |y - ref2|,
+  // |ref2| (4 floats per row); ref2 may alias y (it is read before y is stored)
+  const void* sig_ref; const void* sig_ref2; float* sig_partial; int sig_on;
   const DevState* st; int flag_want;
 };
 cudaError_t ln_mod(const LnArgs& a, cudaStream_t s);
 
 cudaError_t gate_step(DevState* st, const float* sig_partial, int sig_rows, const float* gate_params,
-                      float thr, int T, int B, int policy, const uint8_t* policy_mask,
-                      float* log, unsigned long long cond_handle, int use_cond, cudaStream_t s);
+                      int gate_kind, float thr, int T, int B, int policy,
+                      const uint8_t* policy_mask, float* log, unsigned long long cond_handle,
+                      int use_cond, cudaStream_t s);
 cudaError_t cache_refresh(const DevState* st, const float* h_img, const float* h_in, float* R,
                           void* m_last, const void* m_cur, long n, long m_n, int m_bf16,
                           int flag_want, cudaStream_t s);

@@ -60,6 +60,7 @@ def test_create_rejects_bad_budget(lib, T, B):
     (dict(tau=0.0), 1),
     (dict(patch_ch=16), 7),
     (dict(n_single=0), 1),         # no blocks
+    (dict(gate_kind=3), 1),        # unknown gate architecture
 ])
 def test_create_rejects_bad_arch(lib, patch, code):
     st, h, msg = _create(lib, configs.get_config("tiny"), 10, 5, **patch)

@@ -281,3 +281,51 @@ def test_attention_against_oracle(nq, nk, heads, dh, simt, lib):
     # P and O are rounded to bf16: allow 2^-7 relative to the output scale
     assert np.max(np.abs(got - ref)) <= 2.0 ** -7 * (np.max(np.abs(ref)) + 1e-3)
     ctx.close()
+
+
+# ---------------------------------------------------------------------------
+# the paper's six-input gates (App. A.2) on all six scalars of Eq. 3
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name,kind", [("flux_small", "flux6"), ("qwen_small", "wan6"),
+                                       ("wan_small", "flux6"), ("tiny_ragged", "wan6")])
+def test_six_input_gate_sample_parity(name, kind, lib):
+    cfg = configs.get_config(name, gate_kind=kind)
+    T, B = cfg["T"], cfg["budgets"][0]
+    inp, got, mask, log, nfe = _gpu_sample(cfg, T, B)
+    assert nfe == B and int(mask.sum()) == B and mask[0] == 1
+    g = synth.make_gate6(cfg["gate_seed"], kind)
+    ref = O.sample(cfg, synth.make_weights(cfg), g, inp, T=T, B=B,
+                   drift_override=_gate_inputs(log),
+                   step_override=[None] + [float(v) for v in log[1:, 13]])
+    assert list(mask) == ref["mask"]
+    tol = TOL[cfg["dtype"]]
+    for t in range(1, T):
+        c = int(log[t, 6])
+        t_last = t - int(log[t, 7])
+        f = O.gate_features6(B, T, c, t, t_last, float(log[t, 2]), float(log[t, 13]))
+        assert [np.float32(v) for v in log[t, 8:11]] == f[:3], t
+        assert O.gate_logit6(f, g) == np.float32(log[t, 3]), t
+        sref = ref["log"][t]["s_traj"][2]
+        assert abs(float(log[t, 13]) - sref) <= max(tol, 1e-6) * max(sref, 1e-3), t
+    rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
+    assert float(np.max(np.abs(got.astype(np.float64) - ref["x"]))) <= tol * rms
+
+
+@pytest.mark.parametrize("kind,n", [("mlp3", 81), ("flux6", 449), ("wan6", 785)])
+def test_load_gate_closed_form_schedules(kind, n, lib):
+    """A loaded gate with zero weights has z = its output bias: z = +1 always computes
+    (front-loaded schedule), z = -1 always reuses (forced tail only)."""
+    cfg = configs.get_config("tiny_ragged", gate_kind=kind)
+    T, B = cfg["T"], 3
+    ctx = bag.create(cfg, T=T, B=B)
+    with pytest.raises(bag.BagError) as ei:
+        ctx.load_gate(np.zeros(n + 1, np.float32))
+    assert ei.value.status == 1
+    for b_out, want in ((1.0, [1] * B + [0] * (T - B)), (-1.0, [1] + [0] * (T - B) + [1] * (B - 1))):
+        theta = np.zeros(n, np.float32)
+        theta[-1] = b_out
+        ctx.load_gate(theta)
+        _, _, m, log, nfe = _gpu_sample(cfg, T, B, ctx=ctx)
+        assert list(m) == want and nfe == B
+        assert np.all(log[1:, 3] == np.float32(b_out))
+    ctx.close()
