@@ -310,6 +310,31 @@ def profile_mode(args):
     ctx.close()
 
 
+def replica_barrier(world):
+    """Barrier across the replicas (no-op for one process)."""
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(value, world, device=None):
+    """The largest per-rank value (the job's time is its slowest replica's); works with
+    any initialised process-group backend (NCCL for GPU tensors, gloo on the CPU)."""
+    if world <= 1:
+        return float(value)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_seconds_per_sample(ms_per_step_max, world):
+    """Whole-job throughput as s/sample: every replica finishes one sample per step, so
+    world samples take the slowest replica's step time."""
+    return ms_per_step_max / 1e3 / world
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -401,8 +426,7 @@ def main():
     torch.cuda.synchronize()
 
     def barrier():
-        if ws > 1:
-            torch.distributed.barrier()
+        replica_barrier(ws)
 
     clocks = Clocks(local)
     clocks.start()
@@ -420,11 +444,8 @@ def main():
     barrier()
     clk = clocks.stop()
     ms = e0.elapsed_time(e1) / args.steps
-    if ws > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
-    s_per_sample = ms / 1e3 / ws  # whole job: ws samples per ms-long step
+    ms = max_over_ranks(ms, ws, dev)
+    s_per_sample = job_seconds_per_sample(ms, ws)
     assert all(n == B for n in nfes), nfes
 
     # end to end through the host-buffer entry point (pinned host memory)
@@ -440,10 +461,7 @@ def main():
         ctx.reset()
         ctx.run_host(xh_np, txth_np, pooledh_np)
     e2e_s = (time.perf_counter() - t0) / e2e_n
-    if ws > 1:
-        t = torch.tensor([e2e_s], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = max_over_ranks(e2e_s, ws, dev)
     h2d = x0.numel() * 4 + txth.numel() * 4 + pooledh.numel() * 4
     d2h = x0.numel() * 4 + T * (bag.LOG_FLOATS * 4 + 1) + 32
 
