@@ -52,7 +52,11 @@ enum { BAG_GATE_MLP3 = 0, BAG_GATE_FLUX6 = 1, BAG_GATE_WAN6 = 2 };
 enum {
   BAG_POLICY_BAG = 0,   /* Algorithm 2: gate decision + the two forced pacing rules */
   BAG_POLICY_FULL = 1,  /* uncached sampling: every step evaluates the network */
-  BAG_POLICY_MASK = 2   /* follow a caller-given mask (static schedule) */
+  BAG_POLICY_MASK = 2,  /* follow a caller-given mask (static schedule) */
+  BAG_POLICY_STATIC_UNIFORM = 3, /* Sec. 3.1 static paradigm: B steps evenly spaced */
+  BAG_POLICY_THRESHOLD = 4       /* Sec. 3.1 online threshold paradigm: compute when the
+                                    drift since the last full step exceeds delta; the
+                                    realised NFE is whatever the rule gives */
 };
 
 /* Backbone shape.  kind SINGLE: n_single single-stream blocks on the joint [text; image]
@@ -131,9 +135,11 @@ bag_status bag_load_gate(bag_ctx* ctx, const float* theta, int n, const float* m
                          const float* sd);
 
 /* Choose the schedule policy (BAG_POLICY_*).  For BAG_POLICY_MASK, host_mask[T] gives
- * the per-step bits (host_mask[0] is ignored: step 0 always computes).  The budget
- * pacing of Algorithm 2 applies only to BAG_POLICY_BAG. */
-bag_status bag_set_policy(bag_ctx* ctx, int policy, const uint8_t* host_mask);
+ * the per-step bits (host_mask[0] is ignored: step 0 always computes).
+ * BAG_POLICY_STATIC_UNIFORM computes steps floor(i T / B), i < B.  BAG_POLICY_THRESHOLD
+ * computes step t >= 1 when the fp32 drift > delta (delta ignored by other policies).
+ * The budget pacing of Algorithm 2 applies only to BAG_POLICY_BAG. */
+bag_status bag_set_policy(bag_ctx* ctx, int policy, const uint8_t* host_mask, float delta);
 
 /* Start a new sample: t = 0, c = 0, cache invalid, sticky device error cleared. */
 bag_status bag_reset(bag_ctx* ctx);

@@ -410,6 +410,21 @@ def pace(gate_bit, B, T, c, t):
     return m
 
 
+def static_uniform_schedule(B, T):
+    """Open-loop schedule mu(B, T) of Sec. 3.1's static paradigm, evenly spaced: the
+    steps floor(i * T / B), i = 0 .. B-1 (step 0 included, B distinct steps)."""
+    m = [0] * T
+    for i in range(B):
+        m[(i * T) // B] = 1
+    return m
+
+
+def threshold_decision(drift, delta):
+    """Online threshold paradigm of Sec. 3.1: m_t = [q_t > delta] with q_t the drift
+    since the last full step, compared in fp32; no budget enters the decision."""
+    return 1 if F32(drift) > F32(delta) else 0
+
+
 def schedule_from_gate_bits(bits, B, T):
     """Mask produced by Algorithm 2 from a sequence of raw gate bits (bits[0] unused)."""
     m = [1]
@@ -439,8 +454,10 @@ def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=Non
            step_override=None):
     """One sample of T Euler steps under Algorithm 2.
 
-    policy         'bag' (gate + pacing), 'full' (uncached: every step computes), or a
-                   list of T mask bits to follow (a static schedule).
+    policy         'bag' (gate + pacing), 'full' (uncached: every step computes),
+                   'uniform' (static evenly spaced schedule of B steps), ('threshold', d)
+                   (online rule drift > d, realised NFE not fixed), or a list of T mask
+                   bits to follow (a static schedule).
     drift_override optional per-step drift values (index t) to feed the gate instead of
                    the oracle's own; used to take the decision on another
                    implementation's logged gate inputs.
@@ -489,6 +506,10 @@ def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=Non
                 full = pace(gbit, B, T, c, t)
             elif policy == "full":
                 full = 1
+            elif policy == "uniform":
+                full = static_uniform_schedule(B, T)[t]
+            elif isinstance(policy, tuple) and policy[0] == "threshold":
+                full = threshold_decision(used, policy[1])
             else:
                 full = int(policy[t])
         rec["full"] = full

@@ -19,7 +19,7 @@ LIB_PATH = os.path.join(_HERE, "libbag.so")
 KIND = {"single": 0, "mmdit": 1, "wan": 2}
 DTYPE = {"f32": 0, "bf16": 1}
 GATE_KIND = {"mlp3": 0, "flux6": 1, "wan6": 2}
-POLICY_BAG, POLICY_FULL, POLICY_MASK = 0, 1, 2
+POLICY_BAG, POLICY_FULL, POLICY_MASK, POLICY_STATIC_UNIFORM, POLICY_THRESHOLD = 0, 1, 2, 3, 4
 LOG_FLOATS = 16
 STATUS = {0: "BAG_OK", 1: "BAG_EINVAL", 2: "BAG_ENOMEM", 3: "BAG_ECUDA", 4: "BAG_EORDER",
           5: "BAG_EDEVICE_TIMEOUT", 6: "BAG_ESTATE", 7: "BAG_EUNSUPPORTED"}
@@ -91,7 +91,7 @@ def load(path=None):
         "bag_last_error": ([_P], ctypes.c_char_p),
         "bag_set_stream": ([_P, _P], _I),
         "bag_load_gate": ([_P, _P, _I, _P, _P], _I),
-        "bag_set_policy": ([_P, _I, _P], _I),
+        "bag_set_policy": ([_P, _I, _P, ctypes.c_float], _I),
         "bag_reset": ([_P], _I),
         "bag_step": ([_P, _P, _I, ctypes.POINTER(Cond), _P, _P], _I),
         "bag_run": ([_P, _P, ctypes.POINTER(Cond), ctypes.POINTER(Stats)], _I),
@@ -179,9 +179,10 @@ class Context:
                                          None if mu_a is None else mu_a.ctypes.data,
                                          None if sd_a is None else sd_a.ctypes.data))
 
-    def set_policy(self, policy, mask=None):
+    def set_policy(self, policy, mask=None, delta=0.0):
         m = None if mask is None else np.ascontiguousarray(mask, np.uint8)
-        self._chk(self.lib.bag_set_policy(self.h, policy, None if m is None else m.ctypes.data))
+        self._chk(self.lib.bag_set_policy(self.h, policy, None if m is None else m.ctypes.data,
+                                          float(delta)))
 
     def reset(self):
         self._chk(self.lib.bag_reset(self.h))

@@ -113,6 +113,7 @@ struct bag_ctx {
   float* d_gate = nullptr;
   float thr = 0.f;
   int policy = BAG_POLICY_BAG;
+  float delta = 0.f;  // threshold of BAG_POLICY_THRESHOLD
   uint8_t* d_pmask = nullptr;
 
   // activations
@@ -894,7 +895,7 @@ static void enq_prefix(Enq& q, int use_cond, unsigned long long handle) {
   q.chk(ln_mod(a, q.s));
   q.pre(BAG_PROF_GATE, 0.0, (double)ctx->ni * 8);
   q.chk(gate_step(ctx->st, ctx->sig_partial, ctx->ni, ctx->d_gate, ctx->arch.gate_kind, ctx->thr, ctx->T, ctx->B,
-                  ctx->policy, ctx->d_pmask, ctx->log, handle, use_cond, q.s));
+                  ctx->policy, ctx->d_pmask, ctx->delta, ctx->log, handle, use_cond, q.s));
 }
 
 static void enq_full(Enq& q, int fw) {
@@ -1470,16 +1471,25 @@ bag_status bag_load_gate(bag_ctx* ctx, const float* theta, int n, const float* m
   return BAG_OK;
 }
 
-bag_status bag_set_policy(bag_ctx* ctx, int policy, const uint8_t* host_mask) {
+bag_status bag_set_policy(bag_ctx* ctx, int policy, const uint8_t* host_mask, float delta) {
   if (!ctx) return BAG_EINVAL;
-  if (policy < 0 || policy > 2) return fail(ctx, BAG_EINVAL, "unknown policy");
-  if (policy == BAG_POLICY_MASK) {
-    if (!host_mask) return fail(ctx, BAG_EINVAL, "mask policy needs host_mask");
-    CK(cudaMemcpyAsync(ctx->d_pmask, host_mask, ctx->T, cudaMemcpyHostToDevice, ctx->stream));
+  if (policy < BAG_POLICY_BAG || policy > BAG_POLICY_THRESHOLD) return fail(ctx, BAG_EINVAL, "unknown policy");
+  if (policy == BAG_POLICY_MASK || policy == BAG_POLICY_STATIC_UNIFORM) {
+    std::vector<uint8_t> m(ctx->T, 0);
+    if (policy == BAG_POLICY_MASK) {
+      if (!host_mask) return fail(ctx, BAG_EINVAL, "mask policy needs host_mask");
+      std::memcpy(m.data(), host_mask, ctx->T);
+    } else {
+      // static paradigm: B steps evenly spaced, floor(i * T / B) for i < B
+      for (int i = 0; i < ctx->B; ++i) m[(long)i * ctx->T / ctx->B] = 1;
+    }
+    CK(cudaMemcpyAsync(ctx->d_pmask, m.data(), ctx->T, cudaMemcpyHostToDevice, ctx->stream));
     CK(cudaStreamSynchronize(ctx->stream));
   }
+  if (policy == BAG_POLICY_THRESHOLD && !(delta == delta)) return fail(ctx, BAG_EINVAL, "delta is NaN");
   ctx->policy = policy;
-  destroy_graph(ctx);  // policy is a kernel argument of the captured gate launch
+  ctx->delta = delta;
+  destroy_graph(ctx);  // policy and delta are kernel arguments of the captured gate launch
   return BAG_OK;
 }
 

@@ -243,7 +243,8 @@ BAG_DEV const float* dense32(const float* p, int out, int in, const float* x, fl
 
 __global__ void gate_kernel(DevState* st, const float* partial, int rows, const float* gp,
                             int kind, float thr, int T, int B, int policy, const uint8_t* pmask,
-                            float* log, cudaGraphConditionalHandle handle, int use_cond) {
+                            float delta, float* log, cudaGraphConditionalHandle handle,
+                            int use_cond) {
   const int lane = threadIdx.x;
   const int t = st->t, c = st->c, t_last = st->t_last;
   float num = 0.f, den = 0.f, num2 = 0.f, den2 = 0.f;
@@ -309,7 +310,9 @@ __global__ void gate_kernel(DevState* st, const float* partial, int rows, const 
       if (B - c == 0) m = 0;      // budget exhausted
     } else if (policy == 1) {     // uncached sampling
       m = 1;
-    } else {                      // caller-given mask
+    } else if (policy == 4) {     // online threshold on the drift, no budget
+      m = drift > delta ? 1 : 0;
+    } else {                      // caller-given or static evenly spaced mask
       m = pmask[t] ? 1 : 0;
     }
   }
@@ -339,9 +342,11 @@ __global__ void gate_kernel(DevState* st, const float* partial, int rows, const 
 
 cudaError_t gate_step(DevState* st, const float* sig_partial, int sig_rows, const float* gate_params,
                       int gate_kind, float thr, int T, int B, int policy, const uint8_t* policy_mask,
-                      float* log, unsigned long long cond_handle, int use_cond, cudaStream_t s) {
+                      float delta, float* log, unsigned long long cond_handle, int use_cond,
+                      cudaStream_t s) {
   gate_kernel<<<1, 32, 0, s>>>(st, sig_partial, sig_rows, gate_params, gate_kind, thr, T, B, policy,
-                               policy_mask, log, (cudaGraphConditionalHandle)cond_handle, use_cond);
+                               policy_mask, delta, log, (cudaGraphConditionalHandle)cond_handle,
+                               use_cond);
   return cudaGetLastError();
 }
 

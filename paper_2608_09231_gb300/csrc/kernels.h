@@ -138,8 +138,8 @@ cudaError_t ln_mod(const LnArgs& a, cudaStream_t s);
 
 cudaError_t gate_step(DevState* st, const float* sig_partial, int sig_rows, const float* gate_params,
                       int gate_kind, float thr, int T, int B, int policy,
-                      const uint8_t* policy_mask, float* log, unsigned long long cond_handle,
-                      int use_cond, cudaStream_t s);
+                      const uint8_t* policy_mask, float delta, float* log,
+                      unsigned long long cond_handle, int use_cond, cudaStream_t s);
 cudaError_t cache_refresh(const DevState* st, const float* h_img, const float* h_in, float* R,
                           void* m_last, const void* m_cur, long n, long m_n, int m_bf16,
                           int flag_want, cudaStream_t s);

@@ -30,14 +30,14 @@ def _dev_inputs(cfg, inp):
     return x, txt, pooled
 
 
-def _gpu_sample(cfg, T, B, tau=0.5, policy=None, mask=None, ctx=None):
+def _gpu_sample(cfg, T, B, tau=0.5, policy=None, mask=None, ctx=None, delta=0.0):
     own = ctx is None
     if own:
         ctx = bag.create(cfg, T=T, B=B, tau=tau)
     inp = synth.make_inputs(cfg)
     x, txt, pooled = _dev_inputs(cfg, inp)
     if policy is not None:
-        ctx.set_policy(policy, mask)
+        ctx.set_policy(policy, mask, delta)
     ctx.reset()
     m, log, nfe = ctx.run(x, txt, pooled)
     torch.cuda.synchronize()
@@ -329,3 +329,28 @@ def test_load_gate_closed_form_schedules(kind, n, lib):
         assert list(m) == want and nfe == B
         assert np.all(log[1:, 3] == np.float32(b_out))
     ctx.close()
+
+
+@pytest.mark.parametrize("name", ["tiny_ragged", "flux_small"])
+def test_static_and_threshold_policies(name, lib):
+    """Sec. 3.1's other two paradigms on the same path: the static evenly spaced schedule
+    and the online threshold rule (schedule bit-exact on the GPU's logged drift)."""
+    cfg = configs.get_config(name)
+    T, B = cfg["T"], cfg["budgets"][0]
+    W, g = synth.make_weights(cfg), synth.make_gate(cfg["gate_seed"])
+    inp, got, m, log, nfe = _gpu_sample(cfg, T, B, policy=bag.POLICY_STATIC_UNIFORM)
+    assert list(m) == O.static_uniform_schedule(B, T) and nfe == B
+    ref = O.sample(cfg, W, g, inp, T=T, B=B, policy="uniform")
+    rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
+    assert float(np.max(np.abs(got - ref["x"]))) <= TOL[cfg["dtype"]] * rms
+    # a threshold between the smallest and largest drift of the run above
+    d = np.sort(log[1:, 2])
+    delta = float(d[len(d) // 2])
+    inp, got, m, log, nfe = _gpu_sample(cfg, T, B, policy=bag.POLICY_THRESHOLD, delta=delta)
+    want = [1] + [O.threshold_decision(float(log[t, 2]), delta) for t in range(1, T)]
+    assert list(m) == want and nfe == sum(want)
+    ref = O.sample(cfg, W, g, inp, T=T, B=B, policy=("threshold", delta),
+                   drift_override=_gate_inputs(log))
+    assert ref["mask"] == want
+    rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
+    assert float(np.max(np.abs(got - ref["x"]))) <= TOL[cfg["dtype"]] * rms

@@ -622,3 +622,29 @@ def test_six_input_gates_spend_exactly_B(kind):
         for rec in r["log"][1:]:
             assert len(rec["features"]) == 6
             assert rec["features"][3] == rec["s_traj"][0]
+
+
+# ---------------------------------------------------------------------------
+# the two other scheduling paradigms of Sec. 3.1 on the same signal path
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("T", [1, 7, 10, 50])
+def test_static_uniform_schedule_closed_form(T):
+    for B in range(1, T + 1):
+        m = O.static_uniform_schedule(B, T)
+        assert sum(m) == B and m[0] == 1
+        on = [t for t in range(T) if m[t]]
+        gaps = {b - a for a, b in zip(on, on[1:])}
+        assert gaps <= {T // B, -(-T // B)}       # spacing floor(T/B) or ceil(T/B)
+    assert O.static_uniform_schedule(5, 50) == [1 if t % 10 == 0 else 0 for t in range(50)]
+
+
+def test_threshold_policy_extremes():
+    """q_t >= 0, so delta < 0 computes every step and a huge delta only step 0; the
+    realised NFE is whatever the rule gives (no budget enters)."""
+    cfg, W, g, inp = _tiny(grid=(1, 4, 4), n_txt=3)
+    r = O.sample(cfg, W, g, inp, T=6, B=2, policy=("threshold", -1.0))
+    assert r["mask"] == [1] * 6 and r["nfe"] == 6
+    r = O.sample(cfg, W, g, inp, T=6, B=2, policy=("threshold", 1e9))
+    assert r["mask"] == [1, 0, 0, 0, 0, 0] and r["nfe"] == 1
+    r = O.sample(cfg, W, g, inp, T=6, B=2, policy="uniform")
+    assert r["mask"] == [1, 0, 0, 1, 0, 0]
