@@ -190,8 +190,9 @@ def measured_traffic(kernel, shape):
     return None
 
 
-def dominant_roofline(recs, peaks, peak_src, cfg_name):
-    """Roofline of the (kernel, shape) group that takes the most event time."""
+def dominant_roofline(recs, peaks, peak_src, cfg_name, f32=False):
+    """Roofline of the (kernel, shape) group that takes the most event time.  fp32
+    configurations run on the CUDA cores; their bound is the fp32 FMA rate."""
     groups = {}
     for r in recs:
         key = (r["kind"], r["m"], r["n"], r["k"])
@@ -203,9 +204,22 @@ def dominant_roofline(recs, peaks, peak_src, cfg_name):
     kind, m, n, k = max(groups, key=lambda q: groups[q]["ms"])
     g = groups[(kind, m, n, k)]
     name = KERNEL_NAMES[kind]
+    if f32 and kind in ("gemm", "attention"):
+        name = {"gemm": "gemm_simt_kernel", "attention": "attn_simt_kernel"}[kind]
     avg_ms = g["ms"] / g["launches"]
     total = sum(v["ms"] for v in groups.values())
     shape = [m, n, k]
+    if g["flops"] > 0 and f32:
+        # fp32 FMA peak from the unit counts and clock: 152 SMs x 128 FMA/clk x 2 flop x
+        # sm_max_mhz (the fp32 configuration is a parity check, not a throughput target)
+        per = g["flops"] / g["launches"]
+        ach = per / (avg_ms * 1e-3) / 1e12
+        peak = 152 * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        return {"bound": "alu", "kernel": name, "shape": shape, "achieved": ach, "peak": peak,
+                "unit": "TFLOP/s", "frac": ach / peak, "traffic": None,
+                "peak_source": "fp32 FMA: 152 SMs x 128 lanes x 2 flop x max SM clock",
+                "launches": g["launches"], "avg_launch_ms": avg_ms, "flops_per_launch": per,
+                "share_of_profiled_time": g["ms"] / total}
     if g["flops"] > 0:
         per = g["flops"] / g["launches"]
         ach = per / (avg_ms * 1e-3) / 1e12
@@ -472,7 +486,7 @@ def main():
     recs = ctx.profile_launches()
     peaks, peak_src = _peaks()
     peak_t = peaks.get("bf16_tflops_sustained", 1700.0)
-    roofline = dominant_roofline(recs, peaks, peak_src, args.config)
+    roofline = dominant_roofline(recs, peaks, peak_src, args.config, f32=cfg["dtype"] == "f32")
     g, a = prof["gemm"], prof["attention"]
     gemm_tflops = g["flops"] / (g["ms"] * 1e-3) / 1e12 if g["ms"] > 0 else 0.0
     attn_tflops = a["flops"] / (a["ms"] * 1e-3) / 1e12 if a["ms"] > 0 else 0.0
