@@ -451,7 +451,7 @@ def to64(W):
 
 
 def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=None,
-           step_override=None):
+           step_override=None, guidance=None):
     """One sample of T Euler steps under Algorithm 2.
 
     policy         'bag' (gate + pacing), 'full' (uncached: every step computes),
@@ -462,6 +462,11 @@ def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=Non
                    the oracle's own; used to take the decision on another
                    implementation's logged gate inputs.
     step_override  likewise for the step-to-step change (six-input gates).
+    guidance       classifier-free guidance scale g (None: no guidance).  Then inputs
+                   also holds "txt_u" / "pooled_u" (the unconditional branch), both
+                   branches share one mask (a step is computed for both or reused for
+                   both, App. A.1), each keeps its own cached residual, the signal is
+                   read on the conditional branch (Eq. 3), and v = v_u + g (v_c - v_u).
     The gate is the 3-input MLP unless gate["kind"] names a six-input gate.
     Returns dict(x=final latent, mask, log=[per-step dict]).
     """
@@ -472,6 +477,10 @@ def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=Non
     x = np.asarray(inputs["x"], np.float64)
     txt = np.asarray(inputs["txt"], np.float64)
     pooled = np.asarray(inputs["pooled"], np.float64)
+    if guidance is not None:
+        txt_u = np.asarray(inputs["txt_u"], np.float64)
+        pooled_u = np.asarray(inputs["pooled_u"], np.float64)
+        R_u = None
     sig = sigma_grid(T)
     thr = gate_threshold(tau)
     c = 0
@@ -513,16 +522,26 @@ def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=Non
             else:
                 full = int(policy[t])
         rec["full"] = full
+        if guidance is not None:
+            vec_u = conditioning(cfg, G, sig[t], pooled_u)
         if full:
             h_out = run_stack(cfg, G, blocks, vec, h_in, txt)
             R = h_out - h_in
+            if guidance is not None:
+                h_out_u = run_stack(cfg, G, blocks, vec_u, h_in, txt_u)
+                R_u = h_out_u - h_in
             m_last = m_t
             t_last = t
             c += 1
         else:
             h_out = h_in + R
+            if guidance is not None:
+                h_out_u = h_in + R_u
         m_prev = m_t
         v = final_layer(G, vec, h_out)
+        if guidance is not None:
+            v_u = final_layer(G, vec_u, h_out_u)
+            v = v_u + guidance * (v - v_u)
         x = x + (sig[t + 1] - sig[t]) * v
         mask.append(full)
         log.append(rec)

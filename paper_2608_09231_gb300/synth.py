@@ -303,7 +303,7 @@ def make_gate_any(gate_seed, kind="mlp3"):
 
 
 # Sample inputs: latent noise, text tokens and pooled vector, all N(0, 1).
-INPUT_KEYS = {"x": 1, "txt": 2, "pooled": 3}
+INPUT_KEYS = {"x": 1, "txt": 2, "pooled": 3, "txt_u": 4, "pooled_u": 5}
 
 
 def make_inputs(cfg, sample_seed=0):
@@ -312,6 +312,10 @@ def make_inputs(cfg, sample_seed=0):
     x = normal(seed, INPUT_KEYS["x"], ni * C, 1.0).reshape(ni, C)
     txt = normal(seed, INPUT_KEYS["txt"], nx * d, 1.0).reshape(nx, d)
     pooled = normal(seed, INPUT_KEYS["pooled"], d, 1.0)
+    # the unconditional branch of classifier-free guidance: its own text and pooled vector
+    txt_u = normal(seed, INPUT_KEYS["txt_u"], nx * d, 1.0).reshape(nx, d)
+    pooled_u = normal(seed, INPUT_KEYS["pooled_u"], d, 1.0)
     if cfg["dtype"] == "bf16":
         txt = bf16_round(txt)
-    return {"x": x, "txt": txt, "pooled": pooled}
+        txt_u = bf16_round(txt_u)
+    return {"x": x, "txt": txt, "pooled": pooled, "txt_u": txt_u, "pooled_u": pooled_u}

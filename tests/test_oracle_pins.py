@@ -648,3 +648,34 @@ def test_threshold_policy_extremes():
     assert r["mask"] == [1, 0, 0, 0, 0, 0] and r["nfe"] == 1
     r = O.sample(cfg, W, g, inp, T=6, B=2, policy="uniform")
     assert r["mask"] == [1, 0, 0, 1, 0, 0]
+
+
+# ---------------------------------------------------------------------------
+# classifier-free guidance with one shared mask (App. A.1)
+# ---------------------------------------------------------------------------
+def test_guidance_special_cases():
+    """g = 1 gives v = v_c (the conditional sampler); identical branches give v = v_c
+    for any g, bit for bit; the shared mask spends exactly B and depends only on the
+    conditional branch's signal."""
+    cfg, W, g, inp = _tiny(grid=(1, 4, 4), n_txt=3)
+    T, B = 6, 3
+    base = O.sample(cfg, W, g, inp, T=T, B=B)
+    one = O.sample(cfg, W, g, inp, T=T, B=B, guidance=1.0)
+    assert one["mask"] == base["mask"]
+    assert np.allclose(one["x"], base["x"], atol=1e-12)
+    same = dict(inp, txt_u=inp["txt"], pooled_u=inp["pooled"])
+    r = O.sample(cfg, W, g, same, T=T, B=B, guidance=4.5)
+    assert np.array_equal(r["x"], base["x"]) and r["mask"] == base["mask"]
+    r = O.sample(cfg, W, g, inp, T=T, B=B, guidance=4.5)
+    assert r["nfe"] == B and r["mask"] == base["mask"]   # decisions read the cond branch
+    assert not np.allclose(r["x"], base["x"], atol=1e-6)
+
+
+def test_guidance_reuse_is_per_branch_residual():
+    """With a stack that adds a step-independent vector per branch, any shared schedule
+    reproduces the uncached guided latent: each branch reuses its own residual."""
+    cfg, W, g, inp = _tiny(grid=(1, 4, 4), n_txt=3)
+    W = _constant_offset_net(cfg, W)
+    full = O.sample(cfg, W, g, inp, T=6, B=6, guidance=3.0)["x"]
+    r = O.sample(cfg, W, g, inp, T=6, B=3, guidance=3.0, policy=[1, 0, 0, 1, 0, 1])
+    assert np.allclose(r["x"], full, atol=1e-12)
