@@ -154,9 +154,11 @@ def run_cpu_oracle(cfg_name, reps, warm):
 
 
 def oracle_s_per_sample(cfg, B, rep):
-    """Extrapolate one oracle sample: B full forwards of the whole stack."""
-    return B * (cfg["n_double"] * rep["double_s"] + cfg["n_single"] * rep["single_s"]
-                + cfg["n_wan"] * rep["wan_s"])
+    """Extrapolate one oracle sample: B full forwards of the whole stack (of both
+    branches under classifier-free guidance)."""
+    branches = 1 if cfg.get("guidance") is None else 2
+    return branches * B * (cfg["n_double"] * rep["double_s"] + cfg["n_single"] * rep["single_s"]
+                           + cfg["n_wan"] * rep["wan_s"])
 
 
 # ---------------------------------------------------------------------------
@@ -305,7 +307,7 @@ def profile_mode(args):
 
     from paper_2608_09231_gb300 import bag, configs, synth
 
-    cfg = configs.get_config(args.config)
+    cfg = configs.get_config(args.config, guidance=args.guidance)
     T = args.T or cfg["T"]
     ctx = bag.create(cfg, T=T, B=args.budget)
     inp = synth.make_inputs(cfg)
@@ -314,7 +316,11 @@ def profile_mode(args):
     if cfg["dtype"] == "bf16":
         txt = txt.to(torch.bfloat16)
     pooled = torch.from_numpy(inp["pooled"]).cuda()
-    mask, _, nfe, prof = ctx.profile_run(x, txt, pooled)
+    unc = ()
+    if args.guidance is not None:
+        unc = (torch.from_numpy(inp["txt_u"]).cuda().to(txt.dtype),
+               torch.from_numpy(inp["pooled_u"]).cuda())
+    mask, _, nfe, prof = ctx.profile_run(x, txt, pooled, *unc)
     torch.cuda.synchronize()
     tot = sum(v["ms"] for v in prof.values())
     print(json.dumps({"mode": "profile", "config": args.config, "T": T, "B": args.budget,
@@ -368,6 +374,8 @@ def main():
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--mode", default="sample", choices=["sample", "block", "profile"])
     ap.add_argument("--T", type=int, default=0, help="profile mode: override the step count")
+    ap.add_argument("--guidance", type=float, default=None,
+                    help="classifier-free guidance scale (two branches, one shared mask)")
     args = ap.parse_args()
     if args.mode == "block":
         block_mode(args)
@@ -378,11 +386,14 @@ def main():
     ws, rank, local = _dist()
 
     from paper_2608_09231_gb300 import configs
-    cfg = configs.get_config(args.config)
+    cfg = configs.get_config(args.config, guidance=args.guidance)
     B, T = args.budget, cfg["T"]
     workload = (f"{args.config}-shaped DiT, {cfg['n_double']} double + {cfg['n_single']} single "
                 f"blocks, d={cfg['hidden']}, {cfg['n_img']} img + {cfg['n_txt']} txt tokens, "
                 f"T={T}, B={B}, batch 1")
+    if args.guidance is not None:
+        workload += (f", classifier-free guidance g={args.guidance:g} (conditional and "
+                     "unconditional branch, one shared mask)")
     config = {"workload": workload, "T": T, "B": B, "n_img": cfg["n_img"], "n_txt": cfg["n_txt"],
               "hidden": cfg["hidden"], "global_batch": ws, "seq_len": cfg["n_img"] + cfg["n_txt"],
               "parallelism": f"replicas x{ws}",
@@ -428,12 +439,16 @@ def main():
     if cfg["dtype"] == "bf16":
         txt = txt.to(torch.bfloat16)
     pooled = torch.from_numpy(inp["pooled"]).to(dev)
+    unc = ()
+    if args.guidance is not None:
+        unc = (torch.from_numpy(inp["txt_u"]).to(dev).to(txt.dtype),
+               torch.from_numpy(inp["pooled_u"]).to(dev))
     x = torch.empty_like(x0)
 
     def one_sample():
         ctx.reset()
         x.copy_(x0)
-        return ctx.run(x, txt, pooled)
+        return ctx.run(x, txt, pooled, *unc)
 
     for _ in range(args.warmup):
         one_sample()
@@ -467,22 +482,27 @@ def main():
     txth = torch.from_numpy(inp["txt"].astype(np.float32)).pin_memory()
     pooledh = torch.from_numpy(inp["pooled"]).pin_memory()
     xh_np, txth_np, pooledh_np = xh.numpy(), txth.numpy(), pooledh.numpy()
+    unch = ()
+    if args.guidance is not None:
+        unch = (torch.from_numpy(inp["txt_u"].astype(np.float32)).pin_memory(),
+                torch.from_numpy(inp["pooled_u"]).pin_memory())
+    unch_np = tuple(t.numpy() for t in unch)
     e2e_n = max(1, min(args.steps, 3))
     barrier()
     t0 = time.perf_counter()
     for _ in range(e2e_n):
         xh_np[...] = inp["x"]
         ctx.reset()
-        ctx.run_host(xh_np, txth_np, pooledh_np)
+        ctx.run_host(xh_np, txth_np, pooledh_np, *unch_np)
     e2e_s = (time.perf_counter() - t0) / e2e_n
     e2e_s = max_over_ranks(e2e_s, ws, dev)
-    h2d = x0.numel() * 4 + txth.numel() * 4 + pooledh.numel() * 4
+    h2d = x0.numel() * 4 + txth.numel() * 4 + pooledh.numel() * 4 + sum(t.numel() * 4 for t in unch)
     d2h = x0.numel() * 4 + T * (bag.LOG_FLOATS * 4 + 1) + 32
 
     # profiled sample: per-launch event timing (not part of the timed value)
     ctx.reset()
     x.copy_(x0)
-    _, _, _, prof = ctx.profile_run(x, txt, pooled)
+    _, _, _, prof = ctx.profile_run(x, txt, pooled, *unc)
     recs = ctx.profile_launches()
     peaks, peak_src = _peaks()
     peak_t = peaks.get("bf16_tflops_sustained", 1700.0)
@@ -515,13 +535,13 @@ def main():
             c2.set_stream(stream.cuda_stream)
             c2.reset()
             x.copy_(x0)
-            c2.run(x, txt, pooled)
+            c2.run(x, txt, pooled, *unc)
             torch.cuda.synchronize()
             f0, f1 = torch.cuda.Event(True), torch.cuda.Event(True)
             f0.record(stream)
             c2.reset()
             x.copy_(x0)
-            c2.run(x, txt, pooled)
+            c2.run(x, txt, pooled, *unc)
             f1.record(stream)
             torch.cuda.synchronize()
             sweep[str(Bs)] = f0.elapsed_time(f1) / 1e3
@@ -546,7 +566,8 @@ def main():
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
                 "higher_is_better": False, "scaling": "weak",
                 "vs_baseline": (s_per_sample / PAPER_S_PER_SAMPLE[B]
-                                if B in PAPER_S_PER_SAMPLE and args.config == "flux" else None),
+                                if B in PAPER_S_PER_SAMPLE and args.config == "flux"
+                                and args.guidance is None else None),
                 "dtype": cfg["dtype"], "data": "synthetic (seeded random weights and inputs)",
                 "config": config, "clocks": clk,
                 "e2e": {"value": e2e_s / ws, "unit": "s/sample", "h2d_bytes_per_step": h2d,

@@ -65,7 +65,12 @@ enum {
  * cross-attention to n_txt context tokens and FFN.  hidden = heads * head_dim;
  * rope_axes split head_dim over the (frame, row, col) axes (entries even, sum =
  * head_dim).  dtype: GEMM/attention operand type (the residual stream, latents, the
- * cached residual and all modulation vectors are fp32 in both cases). */
+ * cached residual and all modulation vectors are fp32 in both cases).
+ * cfg = 1 adds classifier-free guidance: every full step evaluates the stack for a
+ * conditional and an unconditional branch (each its own text, pooled vector and cached
+ * residual), both branches share one mask (a step is computed for both or reused for
+ * both, App. A.1), the trajectory signal is read on the conditional branch (Eq. 3), and
+ * the velocity is v_u + guidance * (v_c - v_u).  cfg = 0 ignores guidance. */
 typedef struct {
   int kind;
   int hidden, heads, mlp;
@@ -78,15 +83,21 @@ typedef struct {
   uint64_t weight_seed, gate_seed;
   float tau;          /* gate cutoff: a step computes when sigmoid(z) > tau (0 < tau < 1) */
   int gate_kind;      /* BAG_GATE_* */
+  int cfg;            /* 0 or 1: classifier-free guidance with a shared mask */
+  float guidance;     /* guidance scale g (finite; used when cfg = 1) */
 } bag_arch;
 
 /* Conditioning of one sample (device pointers, read during bag_step / bag_run).
  * txt: [n_txt, hidden] text tokens (fp32 for BAG_F32 contexts, bf16 for BAG_BF16).
  * pooled: [hidden] fp32 pooled text vector added to the time embedding (ignored for
- * WAN; may be null there). */
+ * WAN; may be null there).  txt_uncond / pooled_uncond: the unconditional branch's,
+ * same layouts; required by cfg contexts (pooled_uncond may be null for WAN), ignored
+ * otherwise. */
 typedef struct {
   const void* txt;
   const float* pooled;
+  const void* txt_uncond;
+  const float* pooled_uncond;
 } bag_cond;
 
 /* Per-sample schedule statistics.  mask / log are optional host arrays supplied by the
@@ -158,12 +169,12 @@ bag_status bag_step(bag_ctx* ctx, const float* x, int t, const bag_cond* cond, f
  * host) receives the schedule after one synchronisation at the end. */
 bag_status bag_run(bag_ctx* ctx, float* x_inout, const bag_cond* cond, bag_stats* stats);
 
-/* Same as bag_run with HOST buffers: copies x (fp32 [n_img, patch_ch]), txt (fp32
- * [n_txt, hidden], converted on device for bf16 contexts) and pooled (fp32 [hidden],
- * may be null for WAN) to the device, runs the sample and copies the result back into
+/* Same as bag_run with HOST buffers: copies x (fp32 [n_img, patch_ch]) and the
+ * conditioning cond_host (every pointer host memory; text fp32 [n_txt, hidden] whatever
+ * the context's dtype, converted on device for bf16 contexts; pooled fp32 [hidden], may
+ * be null for WAN) to the device, runs the sample and copies the result back into
  * x_host.  For pageable memory the copies are synchronous. */
-bag_status bag_run_host(bag_ctx* ctx, float* x_host, const float* txt_host,
-                        const float* pooled_host, bag_stats* stats);
+bag_status bag_run_host(bag_ctx* ctx, float* x_host, const bag_cond* cond_host, bag_stats* stats);
 
 /* ---- inspection and single-operation entry points (tests, benchmarks) ---- */
 

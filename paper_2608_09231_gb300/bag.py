@@ -46,11 +46,12 @@ class Arch(ctypes.Structure):
                 ("patch_ch", ctypes.c_int), ("rope_axes", ctypes.c_int * 3),
                 ("dtype", ctypes.c_int), ("weight_seed", ctypes.c_uint64),
                 ("gate_seed", ctypes.c_uint64), ("tau", ctypes.c_float),
-                ("gate_kind", ctypes.c_int)]
+                ("gate_kind", ctypes.c_int), ("cfg", ctypes.c_int), ("guidance", ctypes.c_float)]
 
 
 class Cond(ctypes.Structure):
-    _fields_ = [("txt", ctypes.c_void_p), ("pooled", ctypes.c_void_p)]
+    _fields_ = [("txt", ctypes.c_void_p), ("pooled", ctypes.c_void_p),
+                ("txt_uncond", ctypes.c_void_p), ("pooled_uncond", ctypes.c_void_p)]
 
 
 class ProfEntry(ctypes.Structure):
@@ -95,7 +96,7 @@ def load(path=None):
         "bag_reset": ([_P], _I),
         "bag_step": ([_P, _P, _I, ctypes.POINTER(Cond), _P, _P], _I),
         "bag_run": ([_P, _P, ctypes.POINTER(Cond), ctypes.POINTER(Stats)], _I),
-        "bag_run_host": ([_P, _P, _P, _P, ctypes.POINTER(Stats)], _I),
+        "bag_run_host": ([_P, _P, ctypes.POINTER(Cond), ctypes.POINTER(Stats)], _I),
         "bag_get_weight": ([_P, _I, ctypes.c_char_p, _P, ctypes.c_size_t], _I),
         "bag_forward_block": ([_P, _I, _I, _P], _I),
         "bag_prepare": ([_P, ctypes.POINTER(Cond)], _I),
@@ -130,11 +131,24 @@ def arch_from_config(cfg, tau=0.5):
     a.weight_seed, a.gate_seed = cfg["weight_seed"], cfg["gate_seed"]
     a.tau = tau
     a.gate_kind = GATE_KIND[cfg.get("gate_kind", "mlp3")]
+    g = cfg.get("guidance")
+    a.cfg = 0 if g is None else 1
+    a.guidance = 0.0 if g is None else float(g)
     return a
 
 
 def _ptr(t):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _dp(t):
+    return None if t is None else t.data_ptr()
+
+
+def _cond(txt, pooled, txt_u=None, pooled_u=None):
+    """Device conditioning (torch tensors; the *_u pair is the unconditional branch of
+    a guided context)."""
+    return Cond(_dp(txt), _dp(pooled), _dp(txt_u), _dp(pooled_u))
 
 
 class Context:
@@ -187,12 +201,12 @@ class Context:
     def reset(self):
         self._chk(self.lib.bag_reset(self.h))
 
-    def prepare(self, txt, pooled):
-        c = Cond(txt.data_ptr(), None if pooled is None else pooled.data_ptr())
+    def prepare(self, txt, pooled, txt_u=None, pooled_u=None):
+        c = _cond(txt, pooled, txt_u, pooled_u)
         self._chk(self.lib.bag_prepare(self.h, ctypes.byref(c)))
 
-    def step(self, x, t, txt, pooled, x_out, flag=None):
-        c = Cond(txt.data_ptr(), None if pooled is None else pooled.data_ptr())
+    def step(self, x, t, txt, pooled, x_out, flag=None, txt_u=None, pooled_u=None):
+        c = _cond(txt, pooled, txt_u, pooled_u)
         self._chk(self.lib.bag_step(self.h, _ptr(x), t, ctypes.byref(c), _ptr(x_out), _ptr(flag)))
 
     def _stats(self):
@@ -202,17 +216,17 @@ class Context:
                   log.ctypes.data_as(ctypes.POINTER(ctypes.c_float)), 0, 0, 0)
         return s, mask, log
 
-    def run(self, x, txt, pooled):
+    def run(self, x, txt, pooled, txt_u=None, pooled_u=None):
         """All T steps in place on device tensor x; returns (mask, log, nfe)."""
-        c = Cond(txt.data_ptr(), None if pooled is None else pooled.data_ptr())
+        c = _cond(txt, pooled, txt_u, pooled_u)
         s, mask, log = self._stats()
         self._chk(self.lib.bag_run(self.h, _ptr(x), ctypes.byref(c), ctypes.byref(s)))
         return mask, log, s.nfe
 
-    def profile_run(self, x, txt, pooled):
+    def profile_run(self, x, txt, pooled, txt_u=None, pooled_u=None):
         """Profiled sample (direct launches with events); returns (mask, log, nfe, prof)
         where prof maps a kernel class to dict(launches, ms, flops, bytes)."""
-        c = Cond(txt.data_ptr(), None if pooled is None else pooled.data_ptr())
+        c = _cond(txt, pooled, txt_u, pooled_u)
         s, mask, log = self._stats()
         out = (ProfEntry * len(PROF_KINDS))()
         self._chk(self.lib.bag_profile_run(self.h, _ptr(x), ctypes.byref(c), ctypes.byref(s), out))
@@ -229,17 +243,14 @@ class Context:
         return [dict(kind=PROF_KINDS[r.kind], m=r.m, n=r.n, k=r.k, ms=r.ms, flops=r.flops,
                      bytes=r.bytes) for r in arr[:n.value]]
 
-    def run_host(self, x, txt, pooled):
+    def run_host(self, x, txt, pooled, txt_u=None, pooled_u=None):
         """All T steps with host numpy buffers (x updated in place); returns (mask, log, nfe)."""
         assert x.dtype == np.float32 and x.flags.c_contiguous
-        txt = np.ascontiguousarray(txt, np.float32)
-        pooled_p = None
-        if pooled is not None:
-            pooled = np.ascontiguousarray(pooled, np.float32)
-            pooled_p = pooled.ctypes.data
+        keep = [None if a is None else np.ascontiguousarray(a, np.float32)
+                for a in (txt, pooled, txt_u, pooled_u)]
+        c = Cond(*[None if a is None else a.ctypes.data for a in keep])
         s, mask, log = self._stats()
-        self._chk(self.lib.bag_run_host(self.h, x.ctypes.data, txt.ctypes.data, pooled_p,
-                                        ctypes.byref(s)))
+        self._chk(self.lib.bag_run_host(self.h, x.ctypes.data, ctypes.byref(c), ctypes.byref(s)))
         return mask, log, s.nfe
 
     def get_weight(self, block, name, n):

@@ -132,6 +132,12 @@ struct bag_ctx {
   float *sin_all = nullptr, *t1o = nullptr, *svec = nullptr;  // fp32 conditioning chain
   __nv_bfloat16* splitbuf = nullptr;  // [T, 2 * max(256, d)] hi|lo halves (bf16 configs)
   float *vec_all = nullptr, *mod_all = nullptr, *wan_shared = nullptr;
+  // classifier-free guidance: the unconditional branch's stream, cached residual, staged
+  // conditioning and modulation (Wan: mod_all_u aliases mod_all, its modulation does not
+  // depend on the text), and the conditional velocity of the current step
+  float *hj_u = nullptr, *R_u = nullptr, *vcond = nullptr;
+  void* txt_stage_u = nullptr;
+  float *pooled_stage_u = nullptr, *vec_all_u = nullptr, *svec_u = nullptr, *mod_all_u = nullptr;
   DevState* st = nullptr;     // sampler state
   DevState* st_op = nullptr;  // state for single-operation calls
   float* log = nullptr;
@@ -231,6 +237,8 @@ static bag_status validate_arch(const bag_arch* a, int T, int B) {
   if (!(a->tau > 0.f && a->tau < 1.f)) return fail(nullptr, BAG_EINVAL, "tau must be in (0, 1)");
   if (a->dtype != BAG_F32 && a->dtype != BAG_BF16) return fail(nullptr, BAG_EINVAL, "dtype");
   if (a->gate_kind < BAG_GATE_MLP3 || a->gate_kind > BAG_GATE_WAN6) return fail(nullptr, BAG_EINVAL, "gate_kind");
+  if (a->cfg != 0 && a->cfg != 1) return fail(nullptr, BAG_EINVAL, "cfg must be 0 or 1");
+  if (a->cfg && !std::isfinite(a->guidance)) return fail(nullptr, BAG_EINVAL, "guidance must be finite");
   return BAG_OK;
 }
 
@@ -514,6 +522,18 @@ static bag_status alloc_activations(bag_ctx* ctx) {
   A.add((void**)&ctx->vec_all, (size_t)T * d * 4);
   A.add((void**)&ctx->mod_all, (size_t)T * ctx->mod_stride * 4);
   if (wan) A.add((void**)&ctx->wan_shared, (size_t)T * 8 * d * 4);
+  if (ctx->arch.cfg) {
+    A.add((void**)&ctx->hj_u, (size_t)rows * d * 4);
+    A.add((void**)&ctx->R_u, (size_t)ni * d * 4);
+    A.add((void**)&ctx->vcond, (size_t)ni * ctx->C * 4);
+    A.add(&ctx->txt_stage_u, (size_t)nx * d * es);
+    if (!wan) {
+      A.add((void**)&ctx->pooled_stage_u, (size_t)d * 4);
+      A.add((void**)&ctx->vec_all_u, (size_t)T * d * 4);
+      A.add((void**)&ctx->svec_u, (size_t)T * d * 4);
+      A.add((void**)&ctx->mod_all_u, (size_t)T * ctx->mod_stride * 4);
+    }
+  }
   A.add((void**)&ctx->st, sizeof(DevState));
   A.add((void**)&ctx->st_op, sizeof(DevState));
   A.add((void**)&ctx->log, (size_t)T * kLogFloats * 4);
@@ -524,6 +544,7 @@ static bag_status alloc_activations(bag_ctx* ctx) {
   if (cudaMalloc(&ctx->aarena, A.off) != cudaSuccess)
     return fail(ctx, BAG_ENOMEM, "activation allocation of " + std::to_string(A.off) + " bytes failed");
   A.bind((char*)ctx->aarena);
+  if (ctx->arch.cfg && wan) ctx->mod_all_u = ctx->mod_all;
   CK(cudaMemset(ctx->aarena, 0, A.off));
   std::vector<float2> tab;
   rope_table(ctx, tab);
@@ -693,14 +714,21 @@ static void enq_attn(Enq& q, const void* Q, const void* K, const void* V, long v
   q.chk(attention(a, ctx->st ? &ctx->st->err : nullptr, q.s));
 }
 
+// Per-branch buffers: br 0 is the conditional (or only) branch, br 1 the unconditional
+// branch of classifier-free guidance.
+static float* br_stream(const bag_ctx* ctx, int br) { return br ? ctx->hj_u : ctx->hj; }
+static const float* br_mod(const bag_ctx* ctx, int br) { return br ? ctx->mod_all_u : ctx->mod_all; }
+static const void* br_txt(const bag_ctx* ctx, int br) { return br ? ctx->txt_stage_u : ctx->txt_stage; }
+static int n_branches(const bag_ctx* ctx) { return ctx->arch.cfg ? 2 : 1; }
+
 // One block of the stack on the stream h (joint [N, d] with text rows first, or the
-// Wan image stream [ni, d]).
-static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw) {
+// Wan image stream [ni, d]) with branch br's modulation and (Wan) context.
+static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int br = 0) {
   bag_ctx* ctx = q.ctx;
   const Block& blk = ctx->blocks[b];
   const long d = ctx->d, F = ctx->F, ldc = d + F;
   const int ni = ctx->ni, nx = ctx->nx, N = ctx->N;
-  const float* mod = ctx->mod_all + blk.mod_off;
+  const float* mod = br_mod(ctx, br) + blk.mod_off;
   const long ms = ctx->mod_stride;
   if (blk.type == BT_SINGLE) {
     enq_ln(q, h, d, ctx->xn, d, N, 0, mod, mod + d, mod, mod + d, st, fw);
@@ -823,7 +851,7 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw) {
     kv.col_base = (int)d;
     kv.rope = nullptr;
     kv.bias = (const float*)blk.w.at("ca_kv_b").p;
-    enq_gemm(q, ctx->txt_stage, d, blk.w.at("ca_kv_w"), d, nx, (int)(2 * d), (int)d, kv);
+    enq_gemm(q, br_txt(ctx, br), d, blk.w.at("ca_kv_w"), d, nx, (int)(2 * d), (int)d, kv);
   }
   enq_attn(q, ctx->qc, ctx->kc, ctx->vtc, ctx->vpad_c, ctx->cat, ldc, ni, nx, st, fw);
   {
@@ -854,8 +882,9 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw) {
   }
 }
 
-static float* img_stream(bag_ctx* ctx) {
-  return ctx->arch.kind == BAG_KIND_WAN ? ctx->hj : ctx->hj + (long)ctx->nx * ctx->d;
+static float* img_stream(bag_ctx* ctx, int br = 0) {
+  float* h = br_stream(ctx, br);
+  return ctx->arch.kind == BAG_KIND_WAN ? h : h + (long)ctx->nx * ctx->d;
 }
 
 static void enq_prefix(Enq& q, int use_cond, unsigned long long handle) {
@@ -898,50 +927,90 @@ static void enq_prefix(Enq& q, int use_cond, unsigned long long handle) {
                   ctx->policy, ctx->d_pmask, ctx->delta, ctx->log, handle, use_cond, q.s));
 }
 
+// Full step: the whole stack for every branch, then each branch's residual is cached
+// (and the conditional branch's signal observable m_t becomes m_last).
 static void enq_full(Enq& q, int fw) {
   bag_ctx* ctx = q.ctx;
   const long d = ctx->d;
-  if (ctx->arch.kind != BAG_KIND_WAN)
-    q.chk(copy_rows_f32(ctx->st, fw, ctx->hj, d, ctx->txt_stage, d, ctx->act_bf16, ctx->nx, (int)d, q.s));
-  for (int b = 0; b < ctx->nblk; ++b) enq_block(q, b, ctx->hj, ctx->st, fw);
-  q.pre(BAG_PROF_CACHE, 0.0, (double)ctx->ni * d * (12.0 + 2.0 * ctx->act_size));
-  q.chk(cache_refresh(ctx->st, img_stream(ctx), ctx->h_in, ctx->R, ctx->m_last, ctx->m_cur,
-                      (long)ctx->ni * d, (long)ctx->ni * d, ctx->act_bf16, fw, q.s));
+  for (int br = 0; br < n_branches(ctx); ++br) {
+    float* h = br_stream(ctx, br);
+    if (ctx->arch.kind != BAG_KIND_WAN)
+      q.chk(copy_rows_f32(ctx->st, fw, h, d, br_txt(ctx, br), d, ctx->act_bf16, ctx->nx, (int)d, q.s));
+    if (br) {  // the patch-embed epilogue filled only the conditional stream's image rows
+      q.pre(BAG_PROF_CACHE, 0.0, (double)ctx->ni * d * 8.0);
+      q.chk(copy_rows_f32(ctx->st, fw, img_stream(ctx, br), d, ctx->h_in, d, 0, ctx->ni, (int)d, q.s));
+    }
+    for (int b = 0; b < ctx->nblk; ++b) enq_block(q, b, h, ctx->st, fw, br);
+    const long m_n = br ? 0 : (long)ctx->ni * d;
+    q.pre(BAG_PROF_CACHE, 0.0, (double)ctx->ni * d * 12.0 + (double)m_n * 2.0 * ctx->act_size);
+    q.chk(cache_refresh(ctx->st, img_stream(ctx, br), ctx->h_in, br ? ctx->R_u : ctx->R, ctx->m_last,
+                        ctx->m_cur, (long)ctx->ni * d, m_n, ctx->act_bf16, fw, q.s));
+  }
 }
 
+// Cached step: every branch adds its own cached residual (one shared mask, App. A.1).
 static void enq_skip(Enq& q, int fw) {
   bag_ctx* ctx = q.ctx;
-  q.pre(BAG_PROF_CACHE, 0.0, (double)ctx->ni * ctx->d * 12.0);
-  q.chk(cache_reuse(ctx->st, img_stream(ctx), ctx->h_in, ctx->R, (long)ctx->ni * ctx->d, fw, q.s));
+  for (int br = 0; br < n_branches(ctx); ++br) {
+    q.pre(BAG_PROF_CACHE, 0.0, (double)ctx->ni * ctx->d * 12.0);
+    q.chk(cache_reuse(ctx->st, img_stream(ctx, br), ctx->h_in, br ? ctx->R_u : ctx->R,
+                      (long)ctx->ni * ctx->d, fw, q.s));
+  }
 }
 
+// Final layer and Euler update.  Under guidance the conditional velocity is stored and
+// the unconditional branch's final GEMM applies v_u + g (v_c - v_u) in its epilogue.
 static void enq_suffix(Enq& q) {
   bag_ctx* ctx = q.ctx;
   const long d = ctx->d;
-  const float* fm = ctx->mod_all + ctx->fmod_off;
-  enq_ln(q, img_stream(ctx), d, ctx->xn, d, ctx->ni, 0, fm, fm + d, fm, fm + d, ctx->st, -1);
-  Epi e = base_epi(ctx, ctx->st, -1);
-  e.kind = EPI_EULER;
-  e.bias = (const float*)ctx->G.at("fin_b").p;
-  e.x = ctx->x;
-  e.xb = ctx->act_bf16 ? ctx->xb : nullptr;
-  e.ldx = ctx->C;
-  e.dsig = ctx->dsig;
-  enq_gemm(q, ctx->xn, d, ctx->G.at("fin_w"), d, ctx->ni, ctx->C, (int)d, e);
+  const int nb = n_branches(ctx);
+  for (int br = 0; br < nb; ++br) {
+    const float* fm = br_mod(ctx, br) + ctx->fmod_off;
+    enq_ln(q, img_stream(ctx, br), d, ctx->xn, d, ctx->ni, 0, fm, fm + d, fm, fm + d, ctx->st, -1);
+    Epi e = base_epi(ctx, ctx->st, -1);
+    e.bias = (const float*)ctx->G.at("fin_b").p;
+    if (br + 1 < nb) {
+      e.kind = EPI_STORE;
+      e.out = ctx->vcond;
+      e.ldo = ctx->C;
+      e.out_bf16 = 0;
+    } else {
+      e.kind = EPI_EULER;
+      e.x = ctx->x;
+      e.xb = ctx->act_bf16 ? ctx->xb : nullptr;
+      e.ldx = ctx->C;
+      e.dsig = ctx->dsig;
+      if (br) {
+        e.vcond = ctx->vcond;
+        e.guidance = ctx->arch.guidance;
+      }
+    }
+    enq_gemm(q, ctx->xn, d, ctx->G.at("fin_w"), d, ctx->ni, ctx->C, (int)d, e);
+  }
   q.chk(advance_step(ctx->st, q.s));
 }
 
 // Per-sample conditioning: time embedding and every modulation vector for all T steps
 // in three GEMMs (the modulation weights are read once per sample).
 static bag_status enq_prepare(bag_ctx* ctx, const bag_cond* cond) {
+  const bool wan = ctx->arch.kind == BAG_KIND_WAN;
   if (!cond || !cond->txt) return fail(ctx, BAG_EINVAL, "cond->txt is null");
-  if (ctx->arch.kind != BAG_KIND_WAN && !cond->pooled) return fail(ctx, BAG_EINVAL, "cond->pooled is null");
+  if (!wan && !cond->pooled) return fail(ctx, BAG_EINVAL, "cond->pooled is null");
+  if (ctx->arch.cfg && !cond->txt_uncond) return fail(ctx, BAG_EINVAL, "cond->txt_uncond is null (cfg context)");
+  if (ctx->arch.cfg && !wan && !cond->pooled_uncond)
+    return fail(ctx, BAG_EINVAL, "cond->pooled_uncond is null (cfg context)");
   const long d = ctx->d;
   cudaStream_t s = ctx->stream;
-  if (cond->txt != ctx->txt_stage)
-    CK(cudaMemcpyAsync(ctx->txt_stage, cond->txt, (size_t)ctx->nx * d * ctx->act_size, cudaMemcpyDeviceToDevice, s));
-  if (ctx->arch.kind != BAG_KIND_WAN && cond->pooled != ctx->pooled_stage)
+  const size_t tbytes = (size_t)ctx->nx * d * ctx->act_size;
+  if (cond->txt != ctx->txt_stage) CK(cudaMemcpyAsync(ctx->txt_stage, cond->txt, tbytes, cudaMemcpyDeviceToDevice, s));
+  if (!wan && cond->pooled != ctx->pooled_stage)
     CK(cudaMemcpyAsync(ctx->pooled_stage, cond->pooled, (size_t)d * 4, cudaMemcpyDeviceToDevice, s));
+  if (ctx->arch.cfg) {
+    if (cond->txt_uncond != ctx->txt_stage_u)
+      CK(cudaMemcpyAsync(ctx->txt_stage_u, cond->txt_uncond, tbytes, cudaMemcpyDeviceToDevice, s));
+    if (!wan && cond->pooled_uncond != ctx->pooled_stage_u)
+      CK(cudaMemcpyAsync(ctx->pooled_stage_u, cond->pooled_uncond, (size_t)d * 4, cudaMemcpyDeviceToDevice, s));
+  }
   long cnt = 0;
   Enq q{ctx, s, &cnt};
   // The conditioning chain stays fp32: for bf16 configs each GEMM takes its fp32
@@ -966,29 +1035,36 @@ static bag_status enq_prepare(bag_ctx* ctx, const bag_cond* cond) {
   e1.ldo = d;
   e1.out_bf16 = 0;
   gemm_f32_act(ctx->sin_all, kTembDim, ctx->G.at("t1_w"), (int)d, e1);
-  Epi e2 = base_epi(ctx, nullptr, -1);
-  e2.kind = EPI_VEC;
-  e2.bias = (const float*)ctx->G.at("t2_b").p;
-  e2.out = ctx->vec_all;
-  e2.ldo = d;
-  e2.addend = ctx->arch.kind == BAG_KIND_WAN ? nullptr : ctx->pooled_stage;
-  e2.out2 = ctx->svec;
-  e2.ldo2 = d;
-  e2.out2_bf16 = 0;
-  gemm_f32_act(ctx->t1o, (int)d, ctx->G.at("t2_w"), (int)d, e2);
-  Epi e3 = base_epi(ctx, nullptr, -1);
-  e3.kind = EPI_STORE;
-  e3.bias = ctx->bmod;
-  e3.out_bf16 = 0;
-  if (ctx->arch.kind == BAG_KIND_WAN) {
-    e3.out = ctx->wan_shared;
-    e3.ldo = 8 * d;
-    gemm_f32_act(ctx->svec, (int)d, ctx->wmod, (int)ctx->n_mod, e3);
-    q.chk(expand_wan_mod(ctx->mod_all, ctx->wan_shared, ctx->wan_tabs, ctx->T, ctx->nblk, (int)d, s));
-  } else {
-    e3.out = ctx->mod_all;
-    e3.ldo = ctx->mod_stride;
-    gemm_f32_act(ctx->svec, (int)d, ctx->wmod, (int)ctx->n_mod, e3);
+  // vec = t2(t1) + pooled and every modulation vector, per branch (the time embedding
+  // t1 is shared; a Wan modulation has no text term, so its unconditional branch
+  // reads the conditional one's)
+  const int nb = wan ? 1 : n_branches(ctx);
+  for (int br = 0; br < nb; ++br) {
+    float* svec = br ? ctx->svec_u : ctx->svec;
+    Epi e2 = base_epi(ctx, nullptr, -1);
+    e2.kind = EPI_VEC;
+    e2.bias = (const float*)ctx->G.at("t2_b").p;
+    e2.out = br ? ctx->vec_all_u : ctx->vec_all;
+    e2.ldo = d;
+    e2.addend = wan ? nullptr : (br ? ctx->pooled_stage_u : ctx->pooled_stage);
+    e2.out2 = svec;
+    e2.ldo2 = d;
+    e2.out2_bf16 = 0;
+    gemm_f32_act(ctx->t1o, (int)d, ctx->G.at("t2_w"), (int)d, e2);
+    Epi e3 = base_epi(ctx, nullptr, -1);
+    e3.kind = EPI_STORE;
+    e3.bias = ctx->bmod;
+    e3.out_bf16 = 0;
+    if (wan) {
+      e3.out = ctx->wan_shared;
+      e3.ldo = 8 * d;
+      gemm_f32_act(svec, (int)d, ctx->wmod, (int)ctx->n_mod, e3);
+      q.chk(expand_wan_mod(ctx->mod_all, ctx->wan_shared, ctx->wan_tabs, ctx->T, ctx->nblk, (int)d, s));
+    } else {
+      e3.out = br ? ctx->mod_all_u : ctx->mod_all;
+      e3.ldo = ctx->mod_stride;
+      gemm_f32_act(svec, (int)d, ctx->wmod, (int)ctx->n_mod, e3);
+    }
   }
   if (q.e != cudaSuccess) return fail(ctx, BAG_ECUDA, std::string("prepare: ") + cudaGetErrorString(q.e));
   ctx->n_prepare = cnt;
@@ -1251,25 +1327,33 @@ static bag_status bag_run_impl(bag_ctx* ctx, float* x_inout, const bag_cond* con
   return BAG_OK;
 }
 
-static bag_status bag_run_host_impl(bag_ctx* ctx, float* x_host, const float* txt_host, const float* pooled_host,
-                        bag_stats* stats) {
+static bag_status bag_run_host_impl(bag_ctx* ctx, float* x_host, const bag_cond* ch, bag_stats* stats) {
   if (!ctx) return BAG_EINVAL;
-  if (!x_host || !txt_host) return fail(ctx, BAG_EINVAL, "host buffer is null");
-  if (ctx->arch.kind != BAG_KIND_WAN && !pooled_host) return fail(ctx, BAG_EINVAL, "pooled is null");
+  const bool wan = ctx->arch.kind == BAG_KIND_WAN;
+  if (!x_host || !ch || !ch->txt) return fail(ctx, BAG_EINVAL, "host buffer is null");
+  if (!wan && !ch->pooled) return fail(ctx, BAG_EINVAL, "pooled is null");
+  if (ctx->arch.cfg && (!ch->txt_uncond || (!wan && !ch->pooled_uncond)))
+    return fail(ctx, BAG_EINVAL, "unconditional text / pooled is null (cfg context)");
   if (ctx->next_t != 0) return fail(ctx, BAG_ESTATE, "bag_run_host needs a fresh sample (bag_reset)");
   const long d = ctx->d;
   const size_t xbytes = (size_t)ctx->ni * ctx->C * 4;
-  // stage: latent into the working buffer, text (fp32) into the scratch then convert
+  // stage: latent into the working buffer, each text (fp32) into the scratch then
+  // converted into its staging buffer
   CK(cudaMemcpyAsync(ctx->x, x_host, xbytes, cudaMemcpyHostToDevice, ctx->stream));
-  CK(cudaMemcpyAsync(ctx->tmp_f32, txt_host, (size_t)ctx->nx * d * 4, cudaMemcpyHostToDevice, ctx->stream));
-  if (pooled_host) CK(cudaMemcpyAsync(ctx->pooled_stage, pooled_host, (size_t)d * 4, cudaMemcpyHostToDevice, ctx->stream));
-  void* txt_dev = ctx->txt_stage;
-  if (ctx->act_bf16)
-    CK(to_bf16((__nv_bfloat16*)ctx->txt_stage, ctx->tmp_f32, (long)ctx->nx * d, ctx->stream));
-  else
-    CK(cudaMemcpyAsync(ctx->txt_stage, ctx->tmp_f32, (size_t)ctx->nx * d * 4, cudaMemcpyDeviceToDevice, ctx->stream));
-  bag_cond cond{txt_dev, ctx->pooled_stage};
-  if (ctx->arch.kind == BAG_KIND_WAN) cond.pooled = nullptr;
+  for (int br = 0; br < n_branches(ctx); ++br) {
+    void* stage = br ? ctx->txt_stage_u : ctx->txt_stage;
+    float* pstage = br ? ctx->pooled_stage_u : ctx->pooled_stage;
+    const float* pooled = (const float*)(br ? ch->pooled_uncond : ch->pooled);
+    CK(cudaMemcpyAsync(ctx->tmp_f32, br ? ch->txt_uncond : ch->txt, (size_t)ctx->nx * d * 4,
+                       cudaMemcpyHostToDevice, ctx->stream));
+    if (!wan) CK(cudaMemcpyAsync(pstage, pooled, (size_t)d * 4, cudaMemcpyHostToDevice, ctx->stream));
+    if (ctx->act_bf16)
+      CK(to_bf16((__nv_bfloat16*)stage, ctx->tmp_f32, (long)ctx->nx * d, ctx->stream));
+    else
+      CK(cudaMemcpyAsync(stage, ctx->tmp_f32, (size_t)ctx->nx * d * 4, cudaMemcpyDeviceToDevice, ctx->stream));
+  }
+  bag_cond cond{ctx->txt_stage, wan ? nullptr : ctx->pooled_stage, ctx->txt_stage_u,
+                wan ? nullptr : ctx->pooled_stage_u};
   CKS(bag_run_impl(ctx, ctx->x, &cond, stats));
   CK(cudaMemcpyAsync(x_host, ctx->x, xbytes, cudaMemcpyDeviceToHost, ctx->stream));
   CK(cudaStreamSynchronize(ctx->stream));
@@ -1518,11 +1602,10 @@ bag_status bag_run(bag_ctx* ctx, float* x_inout, const bag_cond* cond, bag_stats
   return leave(ctx, bag_run_impl(ctx, x_inout, cond, stats));
 }
 
-bag_status bag_run_host(bag_ctx* ctx, float* x_host, const float* txt_host, const float* pooled_host,
-                        bag_stats* stats) {
+bag_status bag_run_host(bag_ctx* ctx, float* x_host, const bag_cond* cond_host, bag_stats* stats) {
   if (!ctx) return BAG_EINVAL;
   CKS(enter(ctx));
-  return leave(ctx, bag_run_host_impl(ctx, x_host, txt_host, pooled_host, stats));
+  return leave(ctx, bag_run_host_impl(ctx, x_host, cond_host, stats));
 }
 
 bag_status bag_get_weight(bag_ctx* ctx, int block, const char* name, float* out, size_t n) {

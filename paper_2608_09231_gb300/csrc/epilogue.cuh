@@ -147,6 +147,11 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v) {
     case EPI_EULER: {
       const float ds = e.dsig[t];
       float* x = e.x + (long)row * e.ldx + col0;
+      if (e.vcond) {  // classifier-free guidance: v_u + g (v_c - v_u)
+        const float* vc = e.vcond + (long)row * e.ldx + col0;
+#pragma unroll
+        for (int j = 0; j < NV; ++j) v[j] = v[j] + e.guidance * (vc[j] - v[j]);
+      }
       float nx[NV];
 #pragma unroll
       for (int j = 0; j < NV; ++j) {

@@ -82,6 +82,8 @@ struct Epi {
   __nv_bfloat16* xb = nullptr;
   long ldx = 0;
   const float* dsig = nullptr;  // [T]: sigma_{t+1} - sigma_t
+  const float* vcond = nullptr; // guidance: conditional velocity [rows, ldx]; null = none
+  float guidance = 0.f;         // v = v_u + guidance * (vcond - v_u), v_u this GEMM's output
   // step-dependent addressing and early exit
   const DevState* st = nullptr;  // null: step 0, no flag check
   int flag_want = -1;            // -1: always run; 0/1: run only when st->flag equals it

@@ -37,8 +37,8 @@ def test_library_exports_every_declared_symbol(lib):
     assert sorted(bag.EXPORTS) == _declared()
 
 
-def _create(lib, cfg, T, B, tau=0.5, **patch):
-    a = bag.arch_from_config(cfg, tau)
+def _create(lib, conf, T, B, tau=0.5, **patch):
+    a = bag.arch_from_config(conf, tau)
     for k, v in patch.items():
         setattr(a, k, v)
     h = ctypes.c_void_p()
@@ -61,6 +61,8 @@ def test_create_rejects_bad_budget(lib, T, B):
     (dict(patch_ch=16), 7),
     (dict(n_single=0), 1),         # no blocks
     (dict(gate_kind=3), 1),        # unknown gate architecture
+    (dict(cfg=2), 1),              # guidance flag is 0 or 1
+    (dict(cfg=1, guidance=float("nan")), 1),
 ])
 def test_create_rejects_bad_arch(lib, patch, code):
     st, h, msg = _create(lib, configs.get_config("tiny"), 10, 5, **patch)

@@ -119,3 +119,30 @@ def test_flux_full_size_budget_T_is_uncached(lib):
     ctx.close()
     assert list(ma) == list(mb) == [1] * T
     assert np.array_equal(a, b)
+
+
+def test_full_size_guided_schedule(lib):
+    """Qwen-Image-sized sample under classifier-free guidance (both branches, one mask):
+    NFE = B, m_0 = 1, and the schedule is Algorithm 2 on the gate bits the oracle computes
+    from the logged inputs of the conditional branch."""
+    cfg = configs.get_config("qwen", guidance=4.0)
+    T, B = 50, 10
+    inp = synth.make_inputs(cfg)
+    g = synth.make_gate(cfg["gate_seed"])
+    ctx = bag.create(cfg, T=T, B=B)
+    x = torch.from_numpy(inp["x"].copy()).cuda()
+    txt, pooled = _dev(cfg, inp)
+    txt_u = torch.from_numpy(inp["txt_u"]).cuda().to(torch.bfloat16)
+    pooled_u = torch.from_numpy(inp["pooled_u"]).cuda()
+    ctx.reset()
+    m, log, nfe = ctx.run(x, txt, pooled, txt_u, pooled_u)
+    torch.cuda.synchronize()
+    ctx.close()
+    assert nfe == B and int(m.sum()) == B and m[0] == 1
+    assert np.all(np.isfinite(x.cpu().numpy()))
+    bits = [None]
+    for t in range(1, T):
+        z = O.gate_logit([np.float32(v) for v in log[t, 0:3]], g)
+        assert z == np.float32(log[t, 3])
+        bits.append(1 if z > O.gate_threshold(0.5) else 0)
+    assert list(m) == O.schedule_from_gate_bits(bits, B, T)

@@ -354,3 +354,75 @@ def test_static_and_threshold_policies(name, lib):
     assert ref["mask"] == want
     rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
     assert float(np.max(np.abs(got - ref["x"]))) <= TOL[cfg["dtype"]] * rms
+
+
+# ---------------------------------------------------------------------------
+# classifier-free guidance with one shared mask (App. A.1)
+# ---------------------------------------------------------------------------
+def _dev_uncond(cfg, inp):
+    txt_u = torch.from_numpy(inp["txt_u"]).cuda()
+    if cfg["dtype"] == "bf16":
+        txt_u = txt_u.to(torch.bfloat16)
+    return txt_u, torch.from_numpy(inp["pooled_u"]).cuda()
+
+
+def _gpu_guided(cfg, T, B, inp):
+    ctx = bag.create(cfg, T=T, B=B)
+    x, txt, pooled = _dev_inputs(cfg, inp)
+    txt_u, pooled_u = _dev_uncond(cfg, inp)
+    ctx.reset()
+    m, log, nfe = ctx.run(x, txt, pooled, txt_u, pooled_u)
+    torch.cuda.synchronize()
+    return ctx, x.cpu().numpy(), m, log, nfe
+
+
+@pytest.mark.parametrize("name", ["tiny", "flux_small", "qwen_small", "wan_small"])
+def test_guided_sample_parity(name, lib):
+    """Both branches under one mask, signal on the conditional branch, v = v_u + g (v_c - v_u):
+    schedule bit-exact on the GPU's gate inputs, latent within the dtype's bar; the host
+    entry point gives the same bits as the device one."""
+    g_scale = 4.0
+    cfg = configs.get_config(name, guidance=g_scale)
+    T, B = cfg["T"], cfg["budgets"][0]
+    inp = synth.make_inputs(cfg)
+    ctx, got, mask, log, nfe = _gpu_guided(cfg, T, B, inp)
+    assert nfe == B and int(mask.sum()) == B and mask[0] == 1
+    ctx.reset()
+    xh = inp["x"].astype(np.float32).copy()
+    mh, _, _ = ctx.run_host(xh, inp["txt"], inp["pooled"], inp["txt_u"], inp["pooled_u"])
+    ctx.close()
+    assert list(mh) == list(mask) and np.array_equal(xh, got)
+    W, g = synth.make_weights(cfg), synth.make_gate(cfg["gate_seed"])
+    ref = O.sample(cfg, W, g, inp, T=T, B=B, drift_override=_gate_inputs(log), guidance=g_scale)
+    assert list(mask) == ref["mask"]
+    rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
+    err = float(np.max(np.abs(got.astype(np.float64) - ref["x"])))
+    assert err <= TOL[cfg["dtype"]] * rms, (err, rms)
+    # guidance changed the result (the unconditional branch is not ignored)
+    plain = O.sample(cfg, W, g, inp, T=T, B=B, policy=ref["mask"])
+    assert float(np.max(np.abs(plain["x"] - ref["x"]))) > 10 * err
+
+
+@pytest.mark.parametrize("name", ["tiny", "flux_small", "wan_small"])
+def test_guided_identical_branches_equal_unguided(name, lib):
+    """With the unconditional inputs equal to the conditional ones, v_u = v_c bit for bit,
+    so any guidance scale reproduces the unguided sample exactly."""
+    cfg = configs.get_config(name)
+    T, B = cfg["T"], cfg["budgets"][0]
+    inp, plain, m0, _, _ = _gpu_sample(cfg, T, B)
+    same = dict(inp, txt_u=inp["txt"], pooled_u=inp["pooled"])
+    ctx, got, m1, _, nfe = _gpu_guided(configs.get_config(name, guidance=7.5), T, B, same)
+    ctx.close()
+    assert list(m1) == list(m0) and nfe == B
+    assert np.array_equal(got, plain)
+
+
+def test_guided_context_requires_unconditional_inputs(lib):
+    cfg = configs.get_config("tiny", guidance=2.0)
+    ctx = bag.create(cfg, T=4, B=2)
+    inp = synth.make_inputs(cfg)
+    x, txt, pooled = _dev_inputs(cfg, inp)
+    with pytest.raises(bag.BagError) as ei:
+        ctx.run(x, txt, pooled)
+    assert ei.value.status == 1
+    ctx.close()
