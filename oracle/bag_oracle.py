@@ -49,6 +49,7 @@ import numpy as np
 TEMB_DIM = 256
 ROPE_THETA = 10000.0
 LN_EPS = 1e-6
+RMS_EPS = 1e-6
 
 
 # ---------------------------------------------------------------------------
@@ -160,6 +161,23 @@ def _heads(x, H):
     return x.reshape(x.shape[0], H, -1)
 
 
+def rms_norm_heads(x, w, eps=RMS_EPS):
+    """RMSNorm over each head's channels (FLUX / Qwen-Image QK normalisation):
+    x [N, H, dh] -> x / sqrt(mean over dh of x^2 + eps) * w, w [dh]."""
+    return x / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps) * w
+
+
+def _qk(qkv, d, W, pre, H):
+    """q and k heads of a fused projection [rows, >= 2d] (columns q | k | ...), each
+    RMS-normalised per head when the block carries QK-norm scales (pre + 'q_norm',
+    pre + 'k_norm'); RoPE comes after."""
+    q, k = _heads(qkv[:, :d], H), _heads(qkv[:, d:2 * d], H)
+    if pre + "q_norm" in W:
+        q = rms_norm_heads(q, W[pre + "q_norm"])
+        k = rms_norm_heads(k, W[pre + "k_norm"])
+    return q, k
+
+
 def single_block(h, mod, W, ang, H, rows=None):
     """Single-stream block on the joint sequence h [N, d]; mod = (shift, scale, gate).
 
@@ -171,8 +189,8 @@ def single_block(h, mod, W, ang, H, rows=None):
     xn = modulate(layer_norm(h), shift, scale)
     w1, b1 = W["lin1_w"], W["lin1_b"]
     qkv = linear(xn, w1[:3 * d], b1[:3 * d])
-    q = apply_rope(_heads(qkv[:, :d], H), ang)
-    k = apply_rope(_heads(qkv[:, d:2 * d], H), ang)
+    q, k = _qk(qkv, d, W, "", H)
+    q, k = apply_rope(q, ang), apply_rope(k, ang)
     v = _heads(qkv[:, 2 * d:], H)
     sel = slice(None) if rows is None else rows
     a = attention(q, k, v, q_rows=rows).reshape(-1, d)
@@ -201,8 +219,9 @@ def double_block(img, txt, mod_img, mod_txt, W, ang, H, rows=None):
     qkv_i = linear(modulate(layer_norm(img), mi[0], mi[1]), W["img_qkv_w"], W["img_qkv_b"])
     qkv_t = linear(modulate(layer_norm(txt), mt[0], mt[1]), W["txt_qkv_w"], W["txt_qkv_b"])
     qkv = np.concatenate([qkv_t, qkv_i], axis=0)
-    q = apply_rope(_heads(qkv[:, :d], H), ang)
-    k = apply_rope(_heads(qkv[:, d:2 * d], H), ang)
+    (q_t, k_t), (q_i, k_i) = _qk(qkv_t, d, W, "txt_", H), _qk(qkv_i, d, W, "img_", H)
+    q = apply_rope(np.concatenate([q_t, q_i], axis=0), ang)
+    k = apply_rope(np.concatenate([k_t, k_i], axis=0), ang)
     v = _heads(qkv[:, 2 * d:], H)
     if rows is not None:
         rows = np.asarray(rows)

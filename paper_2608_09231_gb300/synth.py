@@ -158,12 +158,17 @@ GLOBAL_IDS = {
     "pe_w": 0, "pe_b": 1, "t1_w": 2, "t1_b": 3, "t2_w": 4, "t2_b": 5,
     "fmod_w": 6, "fmod_b": 7, "fin_w": 8, "fin_b": 9, "tproj_w": 10, "tproj_b": 11,
 }
-SINGLE_IDS = {"mod_w": 0, "mod_b": 1, "lin1_w": 2, "lin1_b": 3, "lin2_w": 4, "lin2_b": 5}
+SINGLE_IDS = {"mod_w": 0, "mod_b": 1, "lin1_w": 2, "lin1_b": 3, "lin2_w": 4, "lin2_b": 5,
+              "q_norm": 6, "k_norm": 7}
 DOUBLE_IDS = {}
 for _i, _s in enumerate(("img", "txt")):
     for _j, _n in enumerate(("mod", "qkv", "proj", "up", "down")):
         DOUBLE_IDS[f"{_s}_{_n}_w"] = _i * 10 + 2 * _j
         DOUBLE_IDS[f"{_s}_{_n}_b"] = _i * 10 + 2 * _j + 1
+    DOUBLE_IDS[f"{_s}_q_norm"] = 20 + 2 * _i
+    DOUBLE_IDS[f"{_s}_k_norm"] = 21 + 2 * _i
+# QK-norm scales (optional, cfg["qk_norm"]): 1 + N(0, NORM_STD) per head channel.
+NORM_STD = 0.02
 WAN_IDS = {"mod_tab": 0, "sa_qkv_w": 1, "sa_qkv_b": 2, "sa_o_w": 3, "sa_o_b": 4,
            "ca_q_w": 5, "ca_q_b": 6, "ca_kv_w": 7, "ca_kv_b": 8, "ca_o_w": 9, "ca_o_b": 10,
            "ffn_up_w": 11, "ffn_up_b": 12, "ffn_down_w": 13, "ffn_down_b": 14}
@@ -182,9 +187,14 @@ def global_shapes(cfg):
 
 def block_shapes(cfg, btype):
     d, F = cfg["hidden"], cfg["mlp"]
+    qkn = bool(cfg.get("qk_norm"))
+    dh = d // cfg["heads"] if qkn else 0
     if btype == "single":
-        return {"mod_w": (3 * d, d), "mod_b": (3 * d,), "lin1_w": (3 * d + F, d),
-                "lin1_b": (3 * d + F,), "lin2_w": (d, d + F), "lin2_b": (d,)}
+        s = {"mod_w": (3 * d, d), "mod_b": (3 * d,), "lin1_w": (3 * d + F, d),
+             "lin1_b": (3 * d + F,), "lin2_w": (d, d + F), "lin2_b": (d,)}
+        if qkn:
+            s.update({"q_norm": (dh,), "k_norm": (dh,)})
+        return s
     if btype == "double":
         s = {}
         for st in ("img", "txt"):
@@ -193,8 +203,12 @@ def block_shapes(cfg, btype):
                       f"{st}_proj_w": (d, d), f"{st}_proj_b": (d,),
                       f"{st}_up_w": (F, d), f"{st}_up_b": (F,),
                       f"{st}_down_w": (d, F), f"{st}_down_b": (d,)})
+            if qkn:
+                s.update({f"{st}_q_norm": (dh,), f"{st}_k_norm": (dh,)})
         return s
     if btype == "wan":
+        if qkn:
+            raise ValueError("QK-norm is built for single- and double-stream blocks only")
         return {"mod_tab": (6 * d,), "sa_qkv_w": (3 * d, d), "sa_qkv_b": (3 * d,),
                 "sa_o_w": (d, d), "sa_o_b": (d,), "ca_q_w": (d, d), "ca_q_b": (d,),
                 "ca_kv_w": (2 * d, d), "ca_kv_b": (2 * d,), "ca_o_w": (d, d), "ca_o_b": (d,),
@@ -216,6 +230,8 @@ def _ids(btype):
 
 def _gen(cfg, slot, tid, name, shape):
     n = int(np.prod(shape))
+    if name.endswith("_norm"):
+        return np.float32(1.0) + normal(cfg["weight_seed"], slot * 256 + tid, n, NORM_STD).reshape(shape)
     std = BIAS_STD if (name.endswith("_b") or name == "mod_tab") else WEIGHT_STD
     v = normal(cfg["weight_seed"], slot * 256 + tid, n, std).reshape(shape)
     # matrices are stored in the GEMM operand type; biases/tables stay fp32

@@ -315,10 +315,28 @@ def _head_angles(ang, H):
     return [list(a) * 1 for a in ang]
 
 
-def test_single_block_brute_force():
+def _rms_loop(vec, w, eps=1e-6):
+    ms = sum(x * x for x in vec) / len(vec)
+    return [x / math.sqrt(ms + eps) * w[i] for i, x in enumerate(vec)]
+
+
+def _qk_loop(r, off, D, H, W, name, ang_i):
+    """Heads of one projected row at column offset off: RMS-normalised with W[name]
+    (when present) and then rotated."""
+    out = []
+    for hh in range(H):
+        x = r[off + hh * D:off + (hh + 1) * D]
+        if name in W:
+            x = _rms_loop(x, W[name].tolist())
+        out += _rope_loop(x, ang_i)
+    return out
+
+
+@pytest.mark.parametrize("qkn", [False, True])
+def test_single_block_brute_force(qkn):
     rng = np.random.default_rng(3)
     N, d, H, F = 5, 8, 2, 12
-    cfg = {"hidden": d, "mlp": F}
+    cfg = {"hidden": d, "mlp": F, "heads": H, "qk_norm": qkn}
     W = _rand_block(rng, synth.block_shapes(cfg, "single"))
     h = rng.normal(size=(N, d))
     mod = rng.normal(size=3 * d) * 0.5
@@ -329,10 +347,8 @@ def test_single_block_brute_force():
     xn = [[v * (1 + sc[i]) + sh[i] for i, v in enumerate(_ln_loop(list(r)))] for r in h]
     y = _lin_loop(xn, W["lin1_w"].tolist(), W["lin1_b"].tolist())
     D = d // H
-    q = [sum((_rope_loop(r[hh * D:(hh + 1) * D], ang[i]) for hh in range(H)), [])
-         for i, r in enumerate(y)]
-    k = [sum((_rope_loop(r[d + hh * D:d + (hh + 1) * D], ang[i]) for hh in range(H)), [])
-         for i, r in enumerate(y)]
+    q = [_qk_loop(r, 0, D, H, W, "q_norm", ang[i]) for i, r in enumerate(y)]
+    k = [_qk_loop(r, d, D, H, W, "k_norm", ang[i]) for i, r in enumerate(y)]
     v = [r[2 * d:3 * d] for r in y]
     a = _attn_rows(q, k, v, H)
     cat = [a[i] + [_gelu(x) for x in y[i][3 * d:]] for i in range(N)]
@@ -343,10 +359,12 @@ def test_single_block_brute_force():
     assert np.allclose(O.single_block(h, mod, W, ang, H, rows=[4, 1]), got[[4, 1]], atol=1e-13)
 
 
-def test_double_block_brute_force():
+@pytest.mark.parametrize("qkn", [False, True])
+def test_double_block_brute_force(qkn):
     rng = np.random.default_rng(4)
     ni, nx, d, H, F = 4, 3, 8, 2, 12
-    W = _rand_block(rng, synth.block_shapes({"hidden": d, "mlp": F}, "double"))
+    W = _rand_block(rng, synth.block_shapes({"hidden": d, "mlp": F, "heads": H, "qk_norm": qkn},
+                                            "double"))
     img, txt = rng.normal(size=(ni, d)), rng.normal(size=(nx, d))
     mi, mt = rng.normal(size=6 * d) * 0.5, rng.normal(size=6 * d) * 0.5
     pos = np.concatenate([np.zeros((nx, 3)), rng.integers(0, 4, size=(ni, 3))]).astype(float)
@@ -365,10 +383,9 @@ def test_double_block_brute_force():
     qkv_i = _lin_loop(lnmod(img, Mi[0], Mi[1]), W["img_qkv_w"].tolist(), W["img_qkv_b"].tolist())
     joint = qkv_t + qkv_i
     D = d // H
-    q = [sum((_rope_loop(r[hh * D:(hh + 1) * D], ang[i]) for hh in range(H)), [])
-         for i, r in enumerate(joint)]
-    k = [sum((_rope_loop(r[d + hh * D:d + (hh + 1) * D], ang[i]) for hh in range(H)), [])
-         for i, r in enumerate(joint)]
+    pre = ["txt_"] * nx + ["img_"] * ni
+    q = [_qk_loop(r, 0, D, H, W, pre[i] + "q_norm", ang[i]) for i, r in enumerate(joint)]
+    k = [_qk_loop(r, d, D, H, W, pre[i] + "k_norm", ang[i]) for i, r in enumerate(joint)]
     v = [r[2 * d:] for r in joint]
     a = _attn_rows(q, k, v, H)
 
@@ -679,3 +696,47 @@ def test_guidance_reuse_is_per_branch_residual():
     full = O.sample(cfg, W, g, inp, T=6, B=6, guidance=3.0)["x"]
     r = O.sample(cfg, W, g, inp, T=6, B=3, guidance=3.0, policy=[1, 0, 0, 1, 0, 1])
     assert np.allclose(r["x"], full, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# QK-RMSNorm (FLUX / Qwen-Image blocks)
+# ---------------------------------------------------------------------------
+def test_rms_norm_heads_closed_forms():
+    """Unit scale: every head comes out with RMS 1 (up to eps); the result does not
+    depend on the input's scale; for zero-mean heads it equals LayerNorm; the scale
+    multiplies channel by channel."""
+    rng = np.random.default_rng(11)
+    x = rng.normal(size=(6, 3, 16)) * 5
+    y = O.rms_norm_heads(x, np.ones(16), eps=0.0)
+    assert np.allclose(np.sqrt(np.mean(y ** 2, axis=-1)), 1.0, atol=1e-14)
+    assert np.allclose(O.rms_norm_heads(7.5 * x, np.ones(16), eps=0.0), y, atol=1e-13)
+    z = x - x.mean(axis=-1, keepdims=True)
+    assert np.allclose(O.rms_norm_heads(z, np.ones(16)),
+                       O.layer_norm(z.reshape(-1, 16)).reshape(z.shape), atol=1e-12)
+    w = rng.normal(size=16)
+    assert np.allclose(O.rms_norm_heads(x, w, eps=0.0), y * w, atol=1e-13)
+
+
+def test_qk_norm_weights_and_block_use():
+    """The generator's norm scales are 1 + N(0, 0.02) per head channel; a block with unit
+    scales attends with unit-RMS q and k heads; removing the scales gives the plain block."""
+    cfg = configs.get_config("flux_small", qk_norm=True)
+    W = synth.make_weights(cfg, blocks=[0, cfg["n_double"]])
+    b = W["blocks"][0]
+    for n in ("img_q_norm", "img_k_norm", "txt_q_norm", "txt_k_norm"):
+        assert b[n].shape == (cfg["head_dim"],) and abs(float(b[n].mean()) - 1) < 0.01
+    assert 0.01 < float(np.std(b["img_q_norm"])) < 0.03
+    plain = configs.get_config("flux_small")
+    Wp = synth.make_weights(plain, blocks=[0])
+    for n, v in Wp["blocks"][0].items():
+        if n != "type":
+            assert np.array_equal(v, b[n])    # the other tensors are unchanged
+    rng = np.random.default_rng(2)
+    d, H = 8, 2
+    qkv = rng.normal(size=(5, 3 * d)) * 3
+    Wb = {"q_norm": np.ones(d // H), "k_norm": np.ones(d // H)}
+    q, k = O._qk(qkv, d, Wb, "", H)
+    assert np.allclose(np.sqrt(np.mean(q ** 2, axis=-1)), 1.0, atol=1e-6)
+    assert np.allclose(np.sqrt(np.mean(k ** 2, axis=-1)), 1.0, atol=1e-6)
+    q0, k0 = O._qk(qkv, d, {}, "", H)
+    assert np.array_equal(q0, qkv[:, :d].reshape(5, H, -1))
