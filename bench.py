@@ -250,7 +250,7 @@ def block_mode(args):
 
     from paper_2608_09231_gb300 import bag, configs, synth
 
-    cfg = configs.get_config("flux_block")
+    cfg = configs.get_config("flux_block", qk_norm=args.qk_norm)
     d, F, N = cfg["hidden"], cfg["mlp"], cfg["n_img"] + cfg["n_txt"]
     ctx = bag.create(cfg, T=cfg["T"], B=1)
     stream = torch.cuda.current_stream()
@@ -290,7 +290,8 @@ def block_mode(args):
     tf = flops / (ms * 1e-3) / 1e12
     gbs = 12.0 * n / (ms_skip * 1e-3) / 1e9
     print(json.dumps({"mode": "block", "workload": "FLUX-shaped single-stream block, 4096 img + "
-                      "512 txt tokens, d 3072, 24x128 heads, MLP 12288, bf16",
+                      "512 txt tokens, d 3072, 24x128 heads, MLP 12288, bf16"
+                      + (", QK-RMSNorm" if args.qk_norm else ""),
                       "ms_per_block": ms, "block_tflops": tf,
                       "frac_of_bf16_burst": tf / peaks.get("bf16_tflops", 1900.0),
                       "skip_ms": ms_skip, "skip_gbs": gbs,
@@ -307,7 +308,7 @@ def profile_mode(args):
 
     from paper_2608_09231_gb300 import bag, configs, synth
 
-    cfg = configs.get_config(args.config, guidance=args.guidance)
+    cfg = configs.get_config(args.config, guidance=args.guidance, qk_norm=args.qk_norm)
     T = args.T or cfg["T"]
     ctx = bag.create(cfg, T=T, B=args.budget)
     inp = synth.make_inputs(cfg)
@@ -376,6 +377,8 @@ def main():
     ap.add_argument("--T", type=int, default=0, help="profile mode: override the step count")
     ap.add_argument("--guidance", type=float, default=None,
                     help="classifier-free guidance scale (two branches, one shared mask)")
+    ap.add_argument("--qk-norm", action="store_true",
+                    help="per-head RMSNorm of q and k before RoPE (FLUX / Qwen-Image blocks)")
     args = ap.parse_args()
     if args.mode == "block":
         block_mode(args)
@@ -386,7 +389,7 @@ def main():
     ws, rank, local = _dist()
 
     from paper_2608_09231_gb300 import configs
-    cfg = configs.get_config(args.config, guidance=args.guidance)
+    cfg = configs.get_config(args.config, guidance=args.guidance, qk_norm=args.qk_norm)
     B, T = args.budget, cfg["T"]
     workload = (f"{args.config}-shaped DiT, {cfg['n_double']} double + {cfg['n_single']} single "
                 f"blocks, d={cfg['hidden']}, {cfg['n_img']} img + {cfg['n_txt']} txt tokens, "
@@ -394,6 +397,8 @@ def main():
     if args.guidance is not None:
         workload += (f", classifier-free guidance g={args.guidance:g} (conditional and "
                      "unconditional branch, one shared mask)")
+    if args.qk_norm:
+        workload += ", QK-RMSNorm"
     config = {"workload": workload, "T": T, "B": B, "n_img": cfg["n_img"], "n_txt": cfg["n_txt"],
               "hidden": cfg["hidden"], "global_batch": ws, "seq_len": cfg["n_img"] + cfg["n_txt"],
               "parallelism": f"replicas x{ws}",

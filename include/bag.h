@@ -85,6 +85,9 @@ typedef struct {
   int gate_kind;      /* BAG_GATE_* */
   int cfg;            /* 0 or 1: classifier-free guidance with a shared mask */
   float guidance;     /* guidance scale g (finite; used when cfg = 1) */
+  int qk_norm;        /* 0 or 1: RMSNorm of every q and k head (eps 1e-6, learned scale per
+                         head channel) before RoPE, as in FLUX / Qwen-Image blocks; SINGLE
+                         and MMDIT kinds with BAG_BF16 only (else BAG_EUNSUPPORTED) */
 } bag_arch;
 
 /* Conditioning of one sample (device pointers, read during bag_step / bag_run).

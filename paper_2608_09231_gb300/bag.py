@@ -46,7 +46,8 @@ class Arch(ctypes.Structure):
                 ("patch_ch", ctypes.c_int), ("rope_axes", ctypes.c_int * 3),
                 ("dtype", ctypes.c_int), ("weight_seed", ctypes.c_uint64),
                 ("gate_seed", ctypes.c_uint64), ("tau", ctypes.c_float),
-                ("gate_kind", ctypes.c_int), ("cfg", ctypes.c_int), ("guidance", ctypes.c_float)]
+                ("gate_kind", ctypes.c_int), ("cfg", ctypes.c_int), ("guidance", ctypes.c_float),
+                ("qk_norm", ctypes.c_int)]
 
 
 class Cond(ctypes.Structure):
@@ -134,6 +135,7 @@ def arch_from_config(cfg, tau=0.5):
     g = cfg.get("guidance")
     a.cfg = 0 if g is None else 1
     a.guidance = 0.0 if g is None else float(g)
+    a.qk_norm = 1 if cfg.get("qk_norm") else 0
     return a
 
 

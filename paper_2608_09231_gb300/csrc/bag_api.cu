@@ -65,8 +65,9 @@ void sm_uniform(uint64_t seed, uint64_t key, int n, double lo, double hi, float*
 const std::map<std::string, int> kGlobalIds = {
     {"pe_w", 0}, {"pe_b", 1}, {"t1_w", 2}, {"t1_b", 3}, {"t2_w", 4}, {"t2_b", 5},
     {"fmod_w", 6}, {"fmod_b", 7}, {"fin_w", 8}, {"fin_b", 9}, {"tproj_w", 10}, {"tproj_b", 11}};
-const std::map<std::string, int> kSingleIds = {{"mod_w", 0}, {"mod_b", 1}, {"lin1_w", 2},
-                                               {"lin1_b", 3}, {"lin2_w", 4}, {"lin2_b", 5}};
+const std::map<std::string, int> kSingleIds = {{"mod_w", 0},  {"mod_b", 1},  {"lin1_w", 2},
+                                               {"lin1_b", 3}, {"lin2_w", 4}, {"lin2_b", 5},
+                                               {"q_norm", 6}, {"k_norm", 7}};
 std::map<std::string, int> double_ids() {
   std::map<std::string, int> m;
   const char* st[2] = {"img", "txt"};
@@ -76,6 +77,10 @@ std::map<std::string, int> double_ids() {
       m[std::string(st[i]) + "_" + nm[j] + "_w"] = i * 10 + 2 * j;
       m[std::string(st[i]) + "_" + nm[j] + "_b"] = i * 10 + 2 * j + 1;
     }
+  for (int i = 0; i < 2; ++i) {
+    m[std::string(st[i]) + "_q_norm"] = 20 + 2 * i;
+    m[std::string(st[i]) + "_k_norm"] = 21 + 2 * i;
+  }
   return m;
 }
 const std::map<std::string, int> kWanIds = {
@@ -239,6 +244,11 @@ static bag_status validate_arch(const bag_arch* a, int T, int B) {
   if (a->gate_kind < BAG_GATE_MLP3 || a->gate_kind > BAG_GATE_WAN6) return fail(nullptr, BAG_EINVAL, "gate_kind");
   if (a->cfg != 0 && a->cfg != 1) return fail(nullptr, BAG_EINVAL, "cfg must be 0 or 1");
   if (a->cfg && !std::isfinite(a->guidance)) return fail(nullptr, BAG_EINVAL, "guidance must be finite");
+  if (a->qk_norm != 0 && a->qk_norm != 1) return fail(nullptr, BAG_EINVAL, "qk_norm must be 0 or 1");
+  if (a->qk_norm && (a->kind == BAG_KIND_WAN || a->dtype != BAG_BF16))
+    return fail(nullptr, BAG_EUNSUPPORTED, "qk_norm needs a bf16 SINGLE or MMDIT backbone");
+  if (a->qk_norm && a->mlp % dh)
+    return fail(nullptr, BAG_EUNSUPPORTED, "qk_norm needs mlp to be a multiple of head_dim");
   return BAG_OK;
 }
 
@@ -255,10 +265,18 @@ static std::map<std::string, std::vector<long>> global_shapes(const bag_ctx* c) 
 }
 
 static std::map<std::string, std::vector<long>> block_shapes(const bag_ctx* c, int type) {
-  const long d = c->d, F = c->F;
-  if (type == BT_SINGLE)
-    return {{"mod_w", {3 * d, d}}, {"mod_b", {3 * d}}, {"lin1_w", {3 * d + F, d}},
-            {"lin1_b", {3 * d + F}}, {"lin2_w", {d, d + F}}, {"lin2_b", {d}}};
+  const long d = c->d, F = c->F, dh = c->dh;
+  const bool qkn = c->arch.qk_norm != 0;
+  if (type == BT_SINGLE) {
+    std::map<std::string, std::vector<long>> s = {
+        {"mod_w", {3 * d, d}}, {"mod_b", {3 * d}}, {"lin1_w", {3 * d + F, d}},
+        {"lin1_b", {3 * d + F}}, {"lin2_w", {d, d + F}}, {"lin2_b", {d}}};
+    if (qkn) {
+      s["q_norm"] = {dh};
+      s["k_norm"] = {dh};
+    }
+    return s;
+  }
   if (type == BT_DOUBLE) {
     std::map<std::string, std::vector<long>> s;
     for (const char* st : {"img", "txt"}) {
@@ -273,6 +291,10 @@ static std::map<std::string, std::vector<long>> block_shapes(const bag_ctx* c, i
       s[p + "_up_b"] = {F};
       s[p + "_down_w"] = {d, F};
       s[p + "_down_b"] = {d};
+      if (qkn) {
+        s[p + "_q_norm"] = {dh};
+        s[p + "_k_norm"] = {dh};
+      }
     }
     return s;
   }
@@ -396,12 +418,13 @@ static bag_status alloc_weights(bag_ctx* ctx) {
 
 static bag_status seed_weights(bag_ctx* ctx) {
   const uint64_t seed = ctx->arch.weight_seed;
-  auto fill = [&](const Tensor& t, int slot, int id, bool is_bias) -> bag_status {
-    const double sd = 0.02;  // weights and biases N(0, 0.02) (Irwin-Hall(4) approximation)
+  // weights and biases N(0, 0.02) (Irwin-Hall(4) approximation); QK-norm scales
+  // 1 + N(0, 0.02)
+  auto fill = [&](const Tensor& t, int slot, int id, bool is_norm) -> bag_status {
+    const double sd = 0.02;
     const float c32 = (float)(sd * std::sqrt(3.0) / 65536.0);
-    (void)is_bias;
-    cudaError_t e = fill_synth(t.p, t.n, sm_start(seed, (uint64_t)slot * 256 + id), 0, c32, t.bf16,
-                               ctx->stream);
+    cudaError_t e = fill_synth(t.p, t.n, sm_start(seed, (uint64_t)slot * 256 + id), is_norm ? 1.f : 0.f,
+                               c32, t.bf16, ctx->stream);
     if (e != cudaSuccess) return fail(ctx, BAG_ECUDA, std::string("fill: ") + cudaGetErrorString(e));
     return BAG_OK;
   };
@@ -418,7 +441,8 @@ static bag_status seed_weights(bag_ctx* ctx) {
     for (auto& kv : blk.w) {
       auto it = ids.find(kv.first);
       if (it == ids.end()) return fail(ctx, BAG_ESTATE, "unknown block tensor " + kv.first);
-      CKS(fill(kv.second, 1 + b, it->second, false));
+      const bool is_norm = kv.first.size() > 5 && kv.first.compare(kv.first.size() - 5, 5, "_norm") == 0;
+      CKS(fill(kv.second, 1 + b, it->second, is_norm));
     }
   }
   return BAG_OK;
@@ -730,10 +754,18 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int b
   const int ni = ctx->ni, nx = ctx->nx, N = ctx->N;
   const float* mod = br_mod(ctx, br) + blk.mod_off;
   const long ms = ctx->mod_stride;
+  // QK-norm scales of a stream (pre = "", "img_" or "txt_"), when the block has them
+  auto qk_norm = [&](Epi& e, const std::string& pre) {
+    auto it = blk.w.find(pre + "q_norm");
+    if (it == blk.w.end()) return;
+    e.qn_q = (const float*)it->second.p;
+    e.qn_k = (const float*)blk.w.at(pre + "k_norm").p;
+  };
   if (blk.type == BT_SINGLE) {
     enq_ln(q, h, d, ctx->xn, d, N, 0, mod, mod + d, mod, mod + d, st, fw);
     Epi e = base_epi(ctx, st, fw);
     enq_qkv_epi(ctx, e, 0, true);
+    qk_norm(e, "");
     enq_gemm(q, ctx->xn, d, blk.w.at("lin1_w"), d, N, (int)(3 * d + F), (int)d,
              (e.bias = (const float*)blk.w.at("lin1_b").p, e));
     enq_attn(q, ctx->q, ctx->k, ctx->vt, ctx->vpad, ctx->cat, ldc, N, N, st, fw);
@@ -757,9 +789,11 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int b
       Epi e = base_epi(ctx, st, fw);
       enq_qkv_epi(ctx, e, nx, true);
       e.bias = (const float*)blk.w.at("img_qkv_b").p;
+      qk_norm(e, "img_");
       Epi e2 = base_epi(ctx, st, fw);
       enq_qkv_epi(ctx, e2, 0, true);
       e2.bias = (const float*)blk.w.at("txt_qkv_b").p;
+      qk_norm(e2, "txt_");
       enq_gemm2(q, off_act(ctx, ctx->xn, (long)nx * d), d, blk.w.at("img_qkv_w"), d, ni, e,
                 ctx->xn, d, blk.w.at("txt_qkv_w"), d, nx, e2, (int)(3 * d), (int)d);
     }

@@ -522,19 +522,21 @@ cudaError_t to_bf16(__nv_bfloat16* dst, const float* src, long n, cudaStream_t s
 }
 
 // Seeded fill: SplitMix64 stream (state s + (i+1) * golden, finalised by mix), the four
-// 16-bit chunks summed and centred (Irwin-Hall(4)), scaled by c32 in fp32.
+// 16-bit chunks summed and centred (Irwin-Hall(4)), scaled by c32 in fp32, plus an
+// fp32 offset when it is nonzero.
 BAG_DEV uint64_t sm64_mix(uint64_t z) {
   z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
   z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
   return z ^ (z >> 31);
 }
 
-__global__ void fill_synth_kernel(void* dst, long n, uint64_t start, float c32, int bf16) {
+__global__ void fill_synth_kernel(void* dst, long n, uint64_t start, float offset, float c32, int bf16) {
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
     const uint64_t u = sm64_mix(start + (uint64_t)(i + 1) * 0x9E3779B97F4A7C15ull);
     const long q = (long)(u & 0xFFFF) + (long)((u >> 16) & 0xFFFF) + (long)((u >> 32) & 0xFFFF) +
                    (long)(u >> 48) - 131070;
-    const float v = __fmul_rn((float)q, c32);
+    float v = __fmul_rn((float)q, c32);
+    if (offset != 0.f) v = __fadd_rn(offset, v);
     if (bf16)
       reinterpret_cast<__nv_bfloat16*>(dst)[i] = __float2bfloat16_rn(v);
     else
@@ -542,10 +544,10 @@ __global__ void fill_synth_kernel(void* dst, long n, uint64_t start, float c32, 
   }
 }
 
-cudaError_t fill_synth(void* dst, long n, uint64_t start, uint64_t /*unused*/, float c32, int bf16,
+cudaError_t fill_synth(void* dst, long n, uint64_t start, float offset, float c32, int bf16,
                        cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
-  fill_synth_kernel<<<grid_for(n, 256), 256, 0, s>>>(dst, n, start, c32, bf16);
+  fill_synth_kernel<<<grid_for(n, 256), 256, 0, s>>>(dst, n, start, offset, c32, bf16);
   return cudaGetLastError();
 }
 

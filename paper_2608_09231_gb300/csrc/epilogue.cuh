@@ -56,8 +56,10 @@ BAG_DEV void store_vals(void* base, long idx, const float* v, int bf16) {
 // Apply the epilogue to NV consecutive accumulators v[0..NV) of output row `row`,
 // columns [col0, col0 + NV).  NV is even and col0 is a multiple of NV; the chunk never
 // straddles a q/k/v/mlp boundary (those are multiples of 64 columns).
+// rs: EPI_QKV with QK-norm, 1 / RMS of the head that columns col0 .. col0 + NV - 1 of
+// this row belong to (computed by the caller over the whole head).
 template <int NV>
-BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v) {
+BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float rs = 1.f) {
   if (row >= e.M || col0 >= e.N) return;
   if (e.bias) {
 #pragma unroll
@@ -88,6 +90,11 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v) {
       }
       const int jr = row + e.row_off;  // joint-sequence row
       const int cc = lc - region * e.d;
+      if (region < 2 && e.qn_q) {  // per-head RMSNorm of q and k, before the rotation
+        const float* w = (region == 0 ? e.qn_q : e.qn_k) + cc % e.dh;
+#pragma unroll
+        for (int j = 0; j < NV; ++j) v[j] = v[j] * rs * __ldg(w + j);
+      }
       if (region < 2 && e.rope) {
         const int e0 = cc % e.dh;
         const float2* cs = e.rope + (long)jr * (e.dh / 2) + e0 / 2;

@@ -311,11 +311,44 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_after();
       const int row = mt * TC_BM + q * 32 + lane;
       const uint32_t tb = tmem_base + (uint32_t)(acc * BN) + ((uint32_t)(q * 32) << 16);
+      if (e.qn_q) {
+        // QK-norm: the tile holds whole heads (BN a multiple of dh, checked at launch);
+        // a first pass over each q / k head takes its sum of squares (bias included),
+        // the second applies the epilogue with 1 / RMS.  The TMEM loads are warp-wide,
+        // so every lane takes them whatever its row.
+        const int dh = e.dh;
 #pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
-        float v[32];
-        tmem_ld32(tb + (uint32_t)(c * 32), v);
-        epi_apply<32>(e, t, row, nt * BN + c * 32, v);
+        for (int h0 = 0; h0 < BN; h0 += dh) {
+          const int col = nt * BN + h0;
+          float rs = 1.f;
+          if ((col + e.col_base) / e.d < 2 && col < e.N) {
+            float ss = 0.f;
+#pragma unroll 1
+            for (int c = 0; c < dh; c += 32) {
+              float v[32];
+              tmem_ld32(tb + (uint32_t)(h0 + c), v);
+#pragma unroll
+              for (int j = 0; j < 32; ++j) {
+                const float x = v[j] + (e.bias ? __ldg(e.bias + col + c + j) : 0.f);
+                ss = fmaf(x, x, ss);
+              }
+            }
+            rs = rsqrtf(ss / (float)dh + 1e-6f);
+          }
+#pragma unroll 1
+          for (int c = 0; c < dh; c += 32) {
+            float v[32];
+            tmem_ld32(tb + (uint32_t)(h0 + c), v);
+            epi_apply<32>(e, t, row, col + c, v, rs);
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          float v[32];
+          tmem_ld32(tb + (uint32_t)(c * 32), v);
+          epi_apply<32>(e, t, row, nt * BN + c * 32, v);
+        }
       }
       tc_fence_before();
       mbar_arrive(tempty + acc);
@@ -393,10 +426,16 @@ static cudaError_t gemm_tc2(const void* A0, long lda0, const void* W0, long ldw0
   if (a_split && (lda0 < 2L * K || (M1 > 0 && lda1 < 2L * K))) return cudaErrorInvalidValue;
   const int ns = num_sms();
   const int mt = (M0 + TC_BM - 1) / TC_BM + (M1 + TC_BM - 1) / TC_BM;
-  if (N % 256 == 0 && mt * (N / 256) >= ns)
+  // QK-norm epilogues need whole heads in a tile: BN a multiple of dh
+  const bool qkn = e0.qn_q || (M1 > 0 && e1.qn_q);
+  const int min_bn = qkn ? e0.dh : 64;
+  if (qkn && (e0.dh % 32 || (M1 > 0 && e1.dh != e0.dh) || min_bn > 256)) return cudaErrorNotSupported;
+  if (N % 256 == 0 && (mt * (N / 256) >= ns || min_bn > 128))
     return launch_tc<256>(A0, lda0, W0, ldw0, M0, e0, A1, lda1, W1, ldw1, M1, e1, N, K, err, s, a_split);
-  if (N % 128 == 0 && mt * (N / 128) >= ns)
+  if (min_bn > 128) return cudaErrorNotSupported;
+  if (N % 128 == 0 && (mt * (N / 128) >= ns || min_bn > 64))
     return launch_tc<128>(A0, lda0, W0, ldw0, M0, e0, A1, lda1, W1, ldw1, M1, e1, N, K, err, s, a_split);
+  if (min_bn > 64) return cudaErrorNotSupported;
   return launch_tc<64>(A0, lda0, W0, ldw0, M0, e0, A1, lda1, W1, ldw1, M1, e1, N, K, err, s, a_split);
 }
 

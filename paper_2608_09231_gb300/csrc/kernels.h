@@ -82,6 +82,8 @@ struct Epi {
   __nv_bfloat16* xb = nullptr;
   long ldx = 0;
   const float* dsig = nullptr;  // [T]: sigma_{t+1} - sigma_t
+  const float* qn_q = nullptr;  // EPI_QKV: per-head RMSNorm scales [dh] of q and k (both
+  const float* qn_k = nullptr;  //   set or both null), applied before RoPE
   const float* vcond = nullptr; // guidance: conditional velocity [rows, ldx]; null = none
   float guidance = 0.f;         // v = v_u + guidance * (vcond - v_u), v_u this GEMM's output
   // step-dependent addressing and early exit
@@ -154,7 +156,7 @@ cudaError_t sinusoid_all(void* out, int out_bf16, int T, int dim, cudaStream_t s
 cudaError_t expand_wan_mod(float* mod_all, const float* shared6d, const float* tables,
                            int T, int nblocks, int d, cudaStream_t s);
 cudaError_t to_bf16(__nv_bfloat16* dst, const float* src, long n, cudaStream_t s);
-cudaError_t fill_synth(void* dst, long n, uint64_t seed, uint64_t key, float c32, int bf16,
+cudaError_t fill_synth(void* dst, long n, uint64_t start, float offset, float c32, int bf16,
                        cudaStream_t s);
 cudaError_t residual_add(float* out, const float* a, const float* b, long n, cudaStream_t s);
 cudaError_t rel_l1_partials(const void* a, const void* b, int a_bf16, long rows, long cols,

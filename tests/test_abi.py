@@ -63,6 +63,8 @@ def test_create_rejects_bad_budget(lib, T, B):
     (dict(gate_kind=3), 1),        # unknown gate architecture
     (dict(cfg=2), 1),              # guidance flag is 0 or 1
     (dict(cfg=1, guidance=float("nan")), 1),
+    (dict(qk_norm=2), 1),
+    (dict(qk_norm=1), 7),          # QK-norm rides on the tensor-core epilogue: bf16 only
 ])
 def test_create_rejects_bad_arch(lib, patch, code):
     st, h, msg = _create(lib, configs.get_config("tiny"), 10, 5, **patch)
@@ -83,3 +85,8 @@ def test_null_arguments(lib):
     assert lib.bag_reset(None) == 1
     assert lib.bag_run(None, None, None, None) == 1
     lib.bag_destroy(None)
+
+
+def test_qk_norm_unsupported_for_wan(lib):
+    st, h, msg = _create(lib, configs.get_config("wan_small"), 4, 2, qk_norm=1)
+    assert st == 7 and not h.value and "qk_norm" in msg

@@ -39,13 +39,16 @@ def _dev(cfg, inp):
 
 BLOCKS = [
     ("flux_block", {}, [0, 1, 300, 511, 512, 513, 2100, 4607]),
+    ("flux_block", dict(qk_norm=True), [0, 2, 511, 512, 2047, 4607]),
     ("flux", dict(n_double=1, n_single=0), [0, 255, 511, 512, 1000, 3333, 4607]),
+    ("flux", dict(n_double=1, n_single=0, qk_norm=True), [1, 510, 513, 4000]),
     ("qwen", dict(n_double=1), [0, 255, 256, 257, 4000, 7144]),
     ("wan", dict(n_wan=1), [0, 1, 1559, 16000, 32759]),
 ]
 
 
-@pytest.mark.parametrize("name,over,rows", BLOCKS, ids=[b[0] + "-" + str(len(b[1])) for b in BLOCKS])
+@pytest.mark.parametrize("name,over,rows", BLOCKS,
+                         ids=[b[0] + "-" + "-".join(sorted(b[1])) for b in BLOCKS])
 def test_block_full_size_sampled_rows(name, over, rows, lib):
     cfg = configs.get_config(name, **over)
     d = cfg["hidden"]

@@ -426,3 +426,31 @@ def test_guided_context_requires_unconditional_inputs(lib):
         ctx.run(x, txt, pooled)
     assert ei.value.status == 1
     ctx.close()
+
+
+# ---------------------------------------------------------------------------
+# QK-RMSNorm (FLUX / Qwen-Image blocks): fused into the QKV GEMM epilogue
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name", ["single_small", "flux_small", "qwen_small"])
+def test_qk_norm_sample_parity(name, lib):
+    cfg = configs.get_config(name, qk_norm=True)
+    T, B = cfg["T"], cfg["budgets"][0]
+    ctx = bag.create(cfg, T=T, B=B)
+    W = synth.make_weights(cfg)
+    for blk in (0, len(W["blocks"]) - 1):
+        for n in [k for k in W["blocks"][blk] if k.endswith("_norm")]:
+            ref = W["blocks"][blk][n]
+            assert np.array_equal(ctx.get_weight(blk, n, ref.size), ref), (blk, n)
+    inp, got, mask, log, nfe = _gpu_sample(cfg, T, B, ctx=ctx)
+    ctx.close()
+    assert nfe == B and int(mask.sum()) == B
+    g = synth.make_gate(cfg["gate_seed"])
+    ref = O.sample(cfg, W, g, inp, T=T, B=B, drift_override=_gate_inputs(log))
+    assert list(mask) == ref["mask"]
+    rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
+    err = float(np.max(np.abs(got.astype(np.float64) - ref["x"])))
+    assert err <= TOL[cfg["dtype"]] * rms, (err, rms)
+    # the norm changed the result (the scales are not ignored)
+    plain = O.sample(configs.get_config(name), synth.make_weights(configs.get_config(name)), g, inp,
+                     T=T, B=B, policy=ref["mask"])
+    assert float(np.max(np.abs(plain["x"] - ref["x"]))) > 10 * err
