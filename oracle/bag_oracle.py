@@ -92,9 +92,108 @@ def timestep_embedding(tval, dim=TEMB_DIM):
     return np.concatenate([np.cos(args), np.sin(args)])
 
 
-def sigma_grid(T):
-    """Flow-matching noise levels sigma_i = 1 - i/T, i = 0..T (no shift)."""
-    return 1.0 - np.arange(T + 1, dtype=np.float64) / T
+def sigma_grid(T, shift=1.0):
+    """Flow-matching noise levels, i = 0..T: u_i = 1 - i/T, optionally time-shifted
+    sigma_i = s u_i / (1 + (s - 1) u_i) (s = 1: sigma_i = u_i); sigma_0 = 1, sigma_T = 0."""
+    u = 1.0 - np.arange(T + 1, dtype=np.float64) / T
+    if shift == 1.0:
+        return u
+    return shift * u / (1.0 + (shift - 1.0) * u)
+
+
+# ---------------------------------------------------------------------------
+# UniPC (Zhao et al. 2023): the multistep predictor-corrector sampler under which the
+# paper caches Wan2.1 (Sec. 4.1), restated for a flow-matching model
+# ---------------------------------------------------------------------------
+def flow_lambda(sig):
+    """Half log-SNR of x = (1 - sigma) x0 + sigma eps: lambda = log((1 - sigma) / sigma)
+    (-inf at sigma = 1, +inf at sigma = 0)."""
+    sig = np.asarray(sig, np.float64)
+    with np.errstate(divide="ignore"):
+        return np.log1p(-sig) - np.log(sig)
+
+
+class UniPC:
+    """UniPC in its data-prediction form with B(h) = e^{-h} - 1.
+
+    The model's velocity v at (x_i, sigma_i) gives the data prediction m_i = x_i -
+    sigma_i v.  A move from point s to point t (h = lambda_t - lambda_s, alpha = 1 -
+    sigma) is
+
+        x_t = (sigma_t / sigma_s) x_s - alpha_t (e^{-h} - 1) m_s
+              - alpha_t B(h) sum_k rho_k D_k,     D_k = (m_{k} - m_s) / r_k,
+        r_k = (lambda_k - lambda_s) / h,
+
+    over earlier evaluated points k (UniP, the predictor) and, for the corrector UniC,
+    also over the new point t itself (r = 1, D = m_t - m_s).  The rho solve
+    R rho = b with R[j][k] = r_k^j and b_j = j! psi_{j+1} / B(h), where psi_1 = e^{-h} - 1
+    and psi_{j+1} = psi_j / (-h) - 1 / j!.  With one coefficient the fixed value 1/2 is
+    used (order-2 predictor, order-1 corrector), UniPC's simple choice.
+
+    Step i: m_i from the model output; if i > 0 the corrector replaces x_i by UniC from
+    the previous (corrected) sample with the new m_i (the model is not re-evaluated);
+    then the predictor of order p = min(order, i + 1, T - i) (warm-up, first-order last
+    step) gives x_{i+1}.  Earlier points with sigma = 1 (lambda = -inf, their terms
+    vanish in the limit) are not used."""
+
+    def __init__(self, sig, order=2, corrector=True):
+        self.sig = np.asarray(sig, np.float64)
+        self.T = len(self.sig) - 1
+        self.lam = flow_lambda(self.sig)
+        self.order = order
+        self.corrector = corrector
+        self.ms = {}          # step -> data prediction
+        self.x_last = None    # corrected sample of the previous step
+        self.hist_last = []   # history points the previous predictor used
+
+    def _move(self, s, t, x_s, hist, m_t=None):
+        sig, lam = self.sig, self.lam
+        a_t = 1.0 - sig[t]
+        a_s = 1.0 - sig[s]
+        e_mh = (sig[t] * a_s) / (a_t * sig[s])      # e^{-h}, 0 when sigma_s = 1 or sigma_t = 0
+        with np.errstate(divide="ignore"):
+            hh = np.log(e_mh)                       # -h
+        psi = e_mh - 1.0
+        B = psi
+        m_s = self.ms[s]
+        x_t = (sig[t] / sig[s]) * x_s - a_t * psi * m_s
+        rs = [(lam[k] - lam[s]) / (-hh) for k in hist]
+        Ds = [(self.ms[k] - m_s) / r for k, r in zip(hist, rs)]
+        if m_t is not None:
+            rs.append(1.0)
+            Ds.append(m_t - m_s)
+        n = len(Ds)
+        if n == 0:
+            return x_t
+        if n == 1:
+            rho = np.array([0.5])
+        else:
+            b, fact, p = [], 1.0, psi
+            for j in range(1, n + 1):
+                p = (p / hh if np.isfinite(hh) else 0.0) - 1.0 / fact
+                b.append(fact * p / B)
+                fact *= j + 1
+            R = np.array([[r ** j for r in rs] for j in range(n)])
+            rho = np.linalg.solve(R, np.array(b))
+        return x_t - a_t * B * sum(c * D for c, D in zip(rho, Ds))
+
+    def _history(self, s, p):
+        """Up to p - 1 earlier evaluated points before s with sigma < 1."""
+        return [k for k in range(s - 1, s - p, -1) if k >= 0 and self.sig[k] < 1.0]
+
+    def step(self, i, x, v):
+        """Given the sample x_i the model saw and its velocity v_i, return x_{i+1}."""
+        m = x - self.sig[i] * v
+        if i > 0 and self.corrector:
+            self.ms[i] = m
+            x = self._move(i - 1, i, self.x_last, self.hist_last, m_t=m)
+        self.ms[i] = m
+        p = min(self.order, i + 1, self.T - i)
+        hist = self._history(i, p)
+        x_next = self._move(i, i + 1, x, hist)
+        self.x_last = x
+        self.hist_last = hist
+        return x_next
 
 
 # ---------------------------------------------------------------------------
@@ -471,7 +570,9 @@ def to64(W):
 
 def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=None,
            step_override=None, guidance=None):
-    """One sample of T Euler steps under Algorithm 2.
+    """One sample of T sampler steps under Algorithm 2: Euler on the (optionally shifted)
+    sigma grid, or UniPC of order 2 when cfg["sampler"] == "unipc" (cfg["shift"]: the
+    grid's time shift, default 1).
 
     policy         'bag' (gate + pacing), 'full' (uncached: every step computes),
                    'uniform' (static evenly spaced schedule of B steps), ('threshold', d)
@@ -500,7 +601,8 @@ def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=Non
         txt_u = np.asarray(inputs["txt_u"], np.float64)
         pooled_u = np.asarray(inputs["pooled_u"], np.float64)
         R_u = None
-    sig = sigma_grid(T)
+    sig = sigma_grid(T, cfg.get("shift", 1.0))
+    solver = UniPC(sig) if cfg.get("sampler", "euler") == "unipc" else None
     thr = gate_threshold(tau)
     c = 0
     t_last = -1
@@ -561,7 +663,10 @@ def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=Non
         if guidance is not None:
             v_u = final_layer(G, vec_u, h_out_u)
             v = v_u + guidance * (v - v_u)
-        x = x + (sig[t + 1] - sig[t]) * v
+        if solver is not None:
+            x = solver.step(t, x, v)
+        else:
+            x = x + (sig[t + 1] - sig[t]) * v
         mask.append(full)
         log.append(rec)
     return {"x": x, "mask": mask, "log": log, "nfe": c}

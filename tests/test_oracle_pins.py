@@ -740,3 +740,81 @@ def test_qk_norm_weights_and_block_use():
     assert np.allclose(np.sqrt(np.mean(k ** 2, axis=-1)), 1.0, atol=1e-6)
     q0, k0 = O._qk(qkv, d, {}, "", H)
     assert np.array_equal(q0, qkv[:, :d].reshape(5, H, -1))
+
+
+# ---------------------------------------------------------------------------
+# UniPC (the sampler of the paper's Wan runs) and the shifted sigma grid
+# ---------------------------------------------------------------------------
+_S2 = 0.7 ** 2
+
+
+def _gauss_velocity(x, s):
+    """Exact flow-matching velocity for data ~ N(0, 0.7^2) per coordinate."""
+    V = (1 - s) ** 2 * _S2 + s ** 2
+    return (s - (1 - s) * _S2) / V * x
+
+
+def _solve(T, shift, vel, x, **kw):
+    sig = O.sigma_grid(T, shift)
+    if kw.pop("euler", False):
+        for i in range(T):
+            x = x + (sig[i + 1] - sig[i]) * vel(x, sig[i])
+        return x
+    u = O.UniPC(sig, **kw)
+    for i in range(T):
+        x = u.step(i, x, vel(x, sig[i]))
+    return x
+
+
+def test_shifted_sigma_grid():
+    assert np.array_equal(O.sigma_grid(8, 1.0), 1 - np.arange(9) / 8)
+    g = O.sigma_grid(4, 3.0)
+    assert g[0] == 1.0 and g[-1] == 0.0 and np.all(np.diff(g) < 0)
+    assert abs(g[2] - 0.75) < 1e-15          # u = 1/2: 3 u / (1 + 2 u)
+
+
+@pytest.mark.parametrize("shift", [1.0, 5.0])
+def test_unipc_first_order_without_corrector_is_euler(shift):
+    x0 = np.array([1.3, -0.4, 2.0])
+    e = _solve(12, shift, _gauss_velocity, x0, euler=True)
+    u = _solve(12, shift, _gauss_velocity, x0, order=1, corrector=False)
+    assert np.allclose(u, e, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("shift", [1.0, 5.0])
+def test_unipc_exact_for_point_mass_data(shift):
+    """Data concentrated at one point c: every data prediction is c, every difference
+    term vanishes, and the first-order move is the exact flow, so the sampler lands on c."""
+    c = np.array([0.3, -1.1])
+    vel = lambda x, s: (x - c) / s    # noqa: E731
+    for order, corr in ((1, False), (2, True)):
+        x = _solve(9, shift, vel, np.array([2.0, 0.5]), order=order, corrector=corr)
+        assert np.allclose(x, c, atol=1e-12)
+
+
+def test_unipc_convergence_orders_on_gaussian_data():
+    """The probability-flow ODE of N(0, s^2) data maps x(1) to s x(1).  Euler converges at
+    first order; the corrector raises UniPC-1 to second order (UniC adds one order); the
+    order-2 predictor-corrector is at least second order and far more accurate."""
+    x1 = np.array([1.3, -0.4])
+    exact = 0.7 * x1
+
+    def err(T, **kw):
+        return float(np.max(np.abs(_solve(T, 1.0, _gauss_velocity, x1, **kw) - exact)))
+
+    e_eu = [err(T, euler=True) for T in (80, 160)]
+    e_c1 = [err(T, order=1, corrector=True) for T in (80, 160)]
+    e_c2 = [err(T, order=2, corrector=True) for T in (80, 160)]
+    assert 1.9 < e_eu[0] / e_eu[1] < 2.1
+    assert e_c1[0] / e_c1[1] > 3.4
+    assert e_c2[0] / e_c2[1] > 3.6 and e_c2[1] < 0.01 * e_eu[1]
+
+
+def test_unipc_sampler_budget_T_is_uncached_and_differs_from_euler():
+    cfg, W, g, inp = _tiny(grid=(1, 4, 4), n_txt=3)
+    cfg = dict(cfg, sampler="unipc", shift=3.0)
+    a = O.sample(cfg, W, g, inp, T=6, B=6)
+    b = O.sample(cfg, W, g, inp, T=6, B=6, policy="full")
+    assert np.array_equal(a["x"], b["x"])
+    e = O.sample(dict(cfg, sampler="euler"), W, g, inp, T=6, B=6)
+    assert not np.allclose(a["x"], e["x"], atol=1e-6)
