@@ -49,6 +49,13 @@ enum { BAG_F32 = 0, BAG_BF16 = 1 };
  * three) branches 3 -> 8 -> 8 each, concatenated budget-first, 16 -> 32 -> 1 (785
  * params).  Hidden layers use ReLU; the decision is sigmoid(z) > tau. */
 enum { BAG_GATE_MLP3 = 0, BAG_GATE_FLUX6 = 1, BAG_GATE_WAN6 = 2 };
+/* Samplers on the flow-matching noise levels sigma_i (i = 0..T), u_i = 1 - i/T time-shifted
+ * by s: sigma_i = s u_i / (1 + (s - 1) u_i); the model is fed timestep 1000 sigma_i.
+ * EULER: x_{i+1} = x_i + (sigma_{i+1} - sigma_i) v_i.  UNIPC: UniPC (Zhao et al. 2023) of
+ * order 2 with its corrector, in data-prediction form (m = x - sigma v) with
+ * B(h) = e^{-h} - 1, first order at the first and last step; the sampler the paper's Wan
+ * experiments cache (Sec. 4.1).  Its multistep history lives in the context. */
+enum { BAG_SAMPLER_EULER = 0, BAG_SAMPLER_UNIPC = 1 };
 enum {
   BAG_POLICY_BAG = 0,   /* Algorithm 2: gate decision + the two forced pacing rules */
   BAG_POLICY_FULL = 1,  /* uncached sampling: every step evaluates the network */
@@ -88,6 +95,8 @@ typedef struct {
   int qk_norm;        /* 0 or 1: RMSNorm of every q and k head (eps 1e-6, learned scale per
                          head channel) before RoPE, as in FLUX / Qwen-Image blocks; SINGLE
                          and MMDIT kinds with BAG_BF16 only (else BAG_EUNSUPPORTED) */
+  int sampler;        /* BAG_SAMPLER_* */
+  float shift;        /* time shift s of the sigma grid (> 0; 0 is read as 1, no shift) */
 } bag_arch;
 
 /* Conditioning of one sample (device pointers, read during bag_step / bag_run).

@@ -19,6 +19,7 @@ LIB_PATH = os.path.join(_HERE, "libbag.so")
 KIND = {"single": 0, "mmdit": 1, "wan": 2}
 DTYPE = {"f32": 0, "bf16": 1}
 GATE_KIND = {"mlp3": 0, "flux6": 1, "wan6": 2}
+SAMPLER = {"euler": 0, "unipc": 1}
 POLICY_BAG, POLICY_FULL, POLICY_MASK, POLICY_STATIC_UNIFORM, POLICY_THRESHOLD = 0, 1, 2, 3, 4
 LOG_FLOATS = 16
 STATUS = {0: "BAG_OK", 1: "BAG_EINVAL", 2: "BAG_ENOMEM", 3: "BAG_ECUDA", 4: "BAG_EORDER",
@@ -47,7 +48,7 @@ class Arch(ctypes.Structure):
                 ("dtype", ctypes.c_int), ("weight_seed", ctypes.c_uint64),
                 ("gate_seed", ctypes.c_uint64), ("tau", ctypes.c_float),
                 ("gate_kind", ctypes.c_int), ("cfg", ctypes.c_int), ("guidance", ctypes.c_float),
-                ("qk_norm", ctypes.c_int)]
+                ("qk_norm", ctypes.c_int), ("sampler", ctypes.c_int), ("shift", ctypes.c_float)]
 
 
 class Cond(ctypes.Structure):
@@ -136,6 +137,8 @@ def arch_from_config(cfg, tau=0.5):
     a.cfg = 0 if g is None else 1
     a.guidance = 0.0 if g is None else float(g)
     a.qk_norm = 1 if cfg.get("qk_norm") else 0
+    a.sampler = SAMPLER[cfg.get("sampler", "euler")]
+    a.shift = float(cfg.get("shift", 1.0))
     return a
 
 

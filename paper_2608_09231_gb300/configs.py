@@ -51,10 +51,12 @@ _BASE = {
     "qwen": dict(kind="mmdit", hidden=3072, heads=24, mlp=12288, n_double=60, n_single=0,
                  n_wan=0, grid=(1, 83, 83), n_txt=256, patch_ch=64, rope_axes=(16, 56, 56),
                  dtype="bf16", weight_seed=3, gate_seed=103, T=50, budgets=(20, 10)),
-    # Wan2.1-14B-shaped video DiT, 81 frames 480x832 -> 21 x 30 x 52 tokens
+    # Wan2.1-14B-shaped video DiT, 81 frames 480x832 -> 21 x 30 x 52 tokens; sampled with
+    # UniPC as in the paper's Wan runs, on a time-shifted grid (shift 5)
     "wan": dict(kind="wan", hidden=5120, heads=40, mlp=13824, n_double=0, n_single=0,
                 n_wan=40, grid=(21, 30, 52), n_txt=512, patch_ch=64, rope_axes=(44, 42, 42),
-                dtype="bf16", weight_seed=4, gate_seed=104, T=50, budgets=(20,)),
+                dtype="bf16", weight_seed=4, gate_seed=104, T=50, budgets=(20,),
+                sampler="unipc", shift=5.0),
 }
 
 # Reduced variants at which the fp64 oracle runs a whole sample in seconds.  Token
@@ -82,6 +84,8 @@ def get_config(name, **overrides):
         raise KeyError(f"unknown config {name!r}")
     cfg.update(overrides)
     cfg.setdefault("gate_kind", "mlp3")
+    cfg.setdefault("sampler", "euler")     # "euler" or "unipc"
+    cfg.setdefault("shift", 1.0)           # time shift of the sigma grid
     cfg["name"] = name
     d, h = cfg["hidden"], cfg["heads"]
     assert d % h == 0

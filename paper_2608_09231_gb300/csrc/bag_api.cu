@@ -134,6 +134,9 @@ struct bag_ctx {
   float* pooled_stage = nullptr;
   float2* rope = nullptr;
   float* dsig = nullptr;
+  double* d_sigma = nullptr;  // [T + 1] noise levels (time embedding, samplers)
+  float* uni_coef = nullptr;  // UniPC: [T][kUniCoefs]
+  float *uni_xl = nullptr, *uni_m0 = nullptr, *uni_m1 = nullptr;
   float *sin_all = nullptr, *t1o = nullptr, *svec = nullptr;  // fp32 conditioning chain
   __nv_bfloat16* splitbuf = nullptr;  // [T, 2 * max(256, d)] hi|lo halves (bf16 configs)
   float *vec_all = nullptr, *mod_all = nullptr, *wan_shared = nullptr;
@@ -249,6 +252,9 @@ static bag_status validate_arch(const bag_arch* a, int T, int B) {
     return fail(nullptr, BAG_EUNSUPPORTED, "qk_norm needs a bf16 SINGLE or MMDIT backbone");
   if (a->qk_norm && a->mlp % dh)
     return fail(nullptr, BAG_EUNSUPPORTED, "qk_norm needs mlp to be a multiple of head_dim");
+  if (a->sampler != BAG_SAMPLER_EULER && a->sampler != BAG_SAMPLER_UNIPC) return fail(nullptr, BAG_EINVAL, "sampler");
+  if (!(a->shift == 0.f || (std::isfinite(a->shift) && a->shift > 0.f)))
+    return fail(nullptr, BAG_EINVAL, "shift must be positive (0 = no shift)");
   return BAG_OK;
 }
 
@@ -509,6 +515,89 @@ static void rope_table(const bag_ctx* ctx, std::vector<float2>& tab) {
   (void)f;
 }
 
+// Noise levels sigma_i, i = 0..T: u_i = 1 - i/T, time-shifted s u / (1 + (s - 1) u).
+static std::vector<double> sigma_grid(int T, float shift) {
+  const double s = shift == 0.f ? 1.0 : (double)shift;
+  std::vector<double> g(T + 1);
+  for (int i = 0; i <= T; ++i) {
+    const double u = 1.0 - (double)i / T;
+    g[i] = s == 1.0 ? u : s * u / (1.0 + (s - 1.0) * u);
+  }
+  return g;
+}
+
+// UniPC (Zhao et al. 2023) of order 2 with its corrector, data-prediction form with
+// B(h) = e^{-h} - 1, on a flow-matching grid (alpha = 1 - sigma, lambda = log(alpha /
+// sigma)).  A move s -> t is x_t = (sigma_t / sigma_s) x_s - alpha_t psi m_s -
+// alpha_t B sum_k rho_k D_k, psi = B = e^{-h} - 1, D_k = (m_k - m_s) / r_k,
+// r_k = (lambda_k - lambda_s) / h; the corrector adds the new point (r = 1, D = m_t -
+// m_s).  One coefficient: rho = 1/2; two: R rho = b with R = [[1, 1], [r_1, 1]],
+// b_j = j! psi_{j+1} / B, psi_{j+1} = psi_j / (-h) - 1 / j!.  Predictor order
+// min(2, i + 1, T - i); earlier points at sigma = 1 are not used.  The step's update is
+// folded into fixed weights of x_i, the previous corrected sample and m_i, m_{i-1},
+// m_{i-2} (UC_* layout).
+static std::vector<float> unipc_table(const std::vector<double>& sig) {
+  const int T = (int)sig.size() - 1;
+  auto lam = [&](int i) { return std::log1p(-sig[i]) - std::log(sig[i]); };
+  struct Move {
+    double ratio, at, psi, hh;
+  };
+  auto move = [&](int s, int t) {
+    const double at = 1.0 - sig[t], as = 1.0 - sig[s];
+    const double emh = (sig[t] * as) / (at * sig[s]);
+    return Move{sig[t] / sig[s], at, emh - 1.0, std::log(emh)};
+  };
+  std::vector<float> tab((size_t)T * kUniCoefs, 0.f);
+  bool prev_hist = false;  // did the predictor of the previous step use m_{i-2}?
+  for (int i = 0; i < T; ++i) {
+    float* k = tab.data() + (size_t)i * kUniCoefs;
+    k[UC_SIG] = (float)sig[i];
+    if (i == 0) {
+      k[UC_CX] = 1.f;
+    } else {
+      const Move mv = move(i - 1, i);
+      const double B = mv.psi, aB = mv.at * B;
+      double cm1 = -mv.at * mv.psi, cm2 = 0.0, cmt;
+      if (!prev_hist) {
+        cm1 += aB * 0.5;
+        cmt = -aB * 0.5;
+      } else {
+        const double r1 = (lam(i - 2) - lam(i - 1)) / (-mv.hh);
+        double p = mv.psi, b[2];
+        double fact = 1.0;
+        for (int j = 1; j <= 2; ++j) {
+          p = (std::isfinite(mv.hh) ? p / mv.hh : 0.0) - 1.0 / fact;
+          b[j - 1] = fact * p / B;
+          fact *= j + 1;
+        }
+        const double rho1 = (b[0] - b[1]) / (1.0 - r1), rho2 = b[0] - rho1;
+        cm1 += aB * (rho1 / r1 + rho2);
+        cm2 = -aB * rho1 / r1;
+        cmt = -aB * rho2;
+      }
+      k[UC_CLAST] = (float)mv.ratio;
+      k[UC_CM1] = (float)cm1;
+      k[UC_CM2] = (float)cm2;
+      k[UC_CMT] = (float)cmt;
+    }
+    const int p = std::min(std::min(2, i + 1), T - i);
+    const bool hist = p >= 2 && sig[i - 1] < 1.0;
+    const Move mv = move(i, i + 1);
+    double dm0 = -mv.at * mv.psi, dm1 = 0.0;
+    if (hist) {
+      const double r = (lam(i - 1) - lam(i)) / (-mv.hh);
+      const double aB = mv.at * mv.psi;
+      dm0 += aB * 0.5 / r;
+      dm1 = -aB * 0.5 / r;
+    }
+    k[UC_DX] = (float)mv.ratio;
+    k[UC_DM0] = (float)dm0;
+    k[UC_DM1] = (float)dm1;
+    prev_hist = hist;
+  }
+  return tab;
+}
+
 static bag_status alloc_activations(bag_ctx* ctx) {
   const size_t es = ctx->act_size;
   const long d = ctx->d, F = ctx->F, ni = ctx->ni, nx = ctx->nx, N = ctx->N, T = ctx->T;
@@ -539,6 +628,13 @@ static bag_status alloc_activations(bag_ctx* ctx) {
   A.add((void**)&ctx->pooled_stage, (size_t)d * 4);
   A.add((void**)&ctx->rope, (size_t)ctx->nrope * (ctx->dh / 2) * sizeof(float2));
   A.add((void**)&ctx->dsig, (size_t)T * 4);
+  A.add((void**)&ctx->d_sigma, (size_t)(T + 1) * 8);
+  if (ctx->arch.sampler == BAG_SAMPLER_UNIPC) {
+    A.add((void**)&ctx->uni_coef, (size_t)T * kUniCoefs * 4);
+    A.add((void**)&ctx->uni_xl, (size_t)ni * ctx->C * 4);
+    A.add((void**)&ctx->uni_m0, (size_t)ni * ctx->C * 4);
+    A.add((void**)&ctx->uni_m1, (size_t)ni * ctx->C * 4);
+  }
   A.add((void**)&ctx->sin_all, (size_t)T * kTembDim * 4);
   A.add((void**)&ctx->t1o, (size_t)T * d * 4);
   A.add((void**)&ctx->svec, (size_t)T * d * 4);
@@ -573,12 +669,15 @@ static bag_status alloc_activations(bag_ctx* ctx) {
   std::vector<float2> tab;
   rope_table(ctx, tab);
   CK(cudaMemcpy(ctx->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice));
+  const std::vector<double> sg = sigma_grid(T, ctx->arch.shift);
   std::vector<float> ds(T);
-  for (int t = 0; t < T; ++t) {
-    const double s0 = 1.0 - (double)t / T, s1 = 1.0 - (double)(t + 1) / T;
-    ds[t] = (float)(s1 - s0);
-  }
+  for (int t = 0; t < T; ++t) ds[t] = (float)(sg[t + 1] - sg[t]);
   CK(cudaMemcpy(ctx->dsig, ds.data(), T * 4, cudaMemcpyHostToDevice));
+  CK(cudaMemcpy(ctx->d_sigma, sg.data(), (T + 1) * 8, cudaMemcpyHostToDevice));
+  if (ctx->arch.sampler == BAG_SAMPLER_UNIPC) {
+    const std::vector<float> tab = unipc_table(sg);
+    CK(cudaMemcpy(ctx->uni_coef, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice));
+  }
   return BAG_OK;
 }
 
@@ -1018,6 +1117,12 @@ static void enq_suffix(Enq& q) {
         e.vcond = ctx->vcond;
         e.guidance = ctx->arch.guidance;
       }
+      if (ctx->arch.sampler == BAG_SAMPLER_UNIPC) {
+        e.uni_coef = ctx->uni_coef;
+        e.uni_xl = ctx->uni_xl;
+        e.uni_m0 = ctx->uni_m0;
+        e.uni_m1 = ctx->uni_m1;
+      }
     }
     enq_gemm(q, ctx->xn, d, ctx->G.at("fin_w"), d, ctx->ni, ctx->C, (int)d, e);
   }
@@ -1061,7 +1166,7 @@ static bag_status enq_prepare(bag_ctx* ctx, const bag_cond* cond) {
       enq_gemm(q, act, K, W, K, ctx->T, N, K, e);
     }
   };
-  q.chk(sinusoid_all(ctx->sin_all, 0, ctx->T, kTembDim, s));
+  q.chk(sinusoid_all(ctx->sin_all, 0, ctx->d_sigma, ctx->T, kTembDim, s));
   Epi e1 = base_epi(ctx, nullptr, -1);
   e1.kind = EPI_SILU;
   e1.bias = (const float*)ctx->G.at("t1_b").p;

@@ -447,11 +447,11 @@ cudaError_t advance_step(DevState* st, cudaStream_t s) {
 
 // Sinusoidal features of 1000 * sigma_t, sigma_t = 1 - t/T, for every step t < T:
 // [cos(1000 sigma_t f_j), sin(1000 sigma_t f_j)], f_j = exp(-ln(10000) j / (dim/2)).
-__global__ void sinusoid_kernel(void* out, int out_bf16, int T, int dim) {
+__global__ void sinusoid_kernel(void* out, int out_bf16, const double* sigma, int T, int dim) {
   const int t = blockIdx.x, j = threadIdx.x;
   const int half = dim / 2;
   if (t >= T || j >= dim) return;
-  const double sig = 1.0 - (double)t / (double)T;
+  const double sig = sigma[t];
   const int jj = j < half ? j : j - half;
   const double f = exp(-log(10000.0) * (double)jj / (double)half);
   const double arg = 1000.0 * sig * f;
@@ -462,8 +462,8 @@ __global__ void sinusoid_kernel(void* out, int out_bf16, int T, int dim) {
     reinterpret_cast<float*>(out)[(long)t * dim + j] = v;
 }
 
-cudaError_t sinusoid_all(void* out, int out_bf16, int T, int dim, cudaStream_t s) {
-  sinusoid_kernel<<<T, dim, 0, s>>>(out, out_bf16, T, dim);
+cudaError_t sinusoid_all(void* out, int out_bf16, const double* sigma, int T, int dim, cudaStream_t s) {
+  sinusoid_kernel<<<T, dim, 0, s>>>(out, out_bf16, sigma, T, dim);
   return cudaGetLastError();
 }
 

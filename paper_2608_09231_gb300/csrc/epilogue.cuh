@@ -160,10 +160,36 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float r
         for (int j = 0; j < NV; ++j) v[j] = v[j] + e.guidance * (vc[j] - v[j]);
       }
       float nx[NV];
+      if (e.uni_coef) {
+        // UniPC: m_i = x_i - sigma_i v; corrected x_i^c (a combination of x_i, the previous
+        // corrected sample and m_{i-1}, m_{i-2}, m_i); x_{i+1} from x_i^c, m_i, m_{i-1}.
+        // Terms whose weight is zero are not read (uniform across the grid).
+        const float* k = e.uni_coef + (long)t * kUniCoefs;
+        const long idx = (long)row * e.ldx + col0;
+        float* mcur = (t & 1) ? e.uni_m1 : e.uni_m0;        // holds m_{i-2}; receives m_i
+        const float* mprev = (t & 1) ? e.uni_m0 : e.uni_m1;  // m_{i-1}
+        float* xl = e.uni_xl + idx;
+        const bool use_last = k[UC_CLAST] != 0.f, use_m2 = k[UC_CM2] != 0.f;
+        const bool use_m1 = k[UC_CM1] != 0.f || k[UC_DM1] != 0.f;
 #pragma unroll
-      for (int j = 0; j < NV; ++j) {
-        nx[j] = x[j] + ds * v[j];
-        x[j] = nx[j];
+        for (int j = 0; j < NV; ++j) {
+          const float m = x[j] - k[UC_SIG] * v[j];
+          float xc = k[UC_CX] * x[j] + k[UC_CMT] * m;
+          const float m1 = use_m1 ? mprev[idx + j] : 0.f;
+          if (use_last) xc += k[UC_CLAST] * xl[j];
+          if (use_m1) xc += k[UC_CM1] * m1;
+          if (use_m2) xc += k[UC_CM2] * mcur[idx + j];
+          nx[j] = k[UC_DX] * xc + k[UC_DM0] * m + k[UC_DM1] * m1;
+          xl[j] = xc;
+          mcur[idx + j] = m;
+          x[j] = nx[j];
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < NV; ++j) {
+          nx[j] = x[j] + ds * v[j];
+          x[j] = nx[j];
+        }
       }
       if (e.xb) store_vals<NV>(e.xb, (long)row * e.ldx + col0, nx, 1);
       break;

@@ -46,6 +46,10 @@ enum EpiKind : int {
   EPI_DUAL_F32 = 8,   // out = out2 = acc + bias (f32)
 };
 
+// UniPC coefficients per step: sigma_i; corrector weights of x_i, the previous corrected
+// sample, m_{i-1}, m_{i-2}, m_i; predictor weights of the corrected sample, m_i, m_{i-1}.
+enum { UC_SIG = 0, UC_CX, UC_CLAST, UC_CM1, UC_CM2, UC_CMT, UC_DX, UC_DM0, UC_DM1, kUniCoefs };
+
 struct Epi {
   int kind = EPI_STORE;
   int M = 0, N = 0;
@@ -86,6 +90,13 @@ struct Epi {
   const float* qn_k = nullptr;  //   set or both null), applied before RoPE
   const float* vcond = nullptr; // guidance: conditional velocity [rows, ldx]; null = none
   float guidance = 0.f;         // v = v_u + guidance * (vcond - v_u), v_u this GEMM's output
+  // EPI_EULER as a UniPC step when uni_coef is set: per step kUniCoefs coefficients,
+  // the previous corrected sample uni_xl and the data predictions of the last two
+  // steps in uni_m[step & 1] (all fp32 [rows, ldx])
+  const float* uni_coef = nullptr;
+  float* uni_xl = nullptr;
+  float* uni_m0 = nullptr;
+  float* uni_m1 = nullptr;
   // step-dependent addressing and early exit
   const DevState* st = nullptr;  // null: step 0, no flag check
   int flag_want = -1;            // -1: always run; 0/1: run only when st->flag equals it
@@ -152,7 +163,7 @@ cudaError_t cache_reuse(const DevState* st, float* h_img, const float* h_in, con
 cudaError_t copy_rows_f32(const DevState* st, int flag_want, float* dst, long ldd, const void* src,
                           long lds, int src_bf16, int rows, int cols, cudaStream_t s);
 cudaError_t advance_step(DevState* st, cudaStream_t s);
-cudaError_t sinusoid_all(void* out, int out_bf16, int T, int dim, cudaStream_t s);
+cudaError_t sinusoid_all(void* out, int out_bf16, const double* sigma, int T, int dim, cudaStream_t s);
 cudaError_t expand_wan_mod(float* mod_all, const float* shared6d, const float* tables,
                            int T, int nblocks, int d, cudaStream_t s);
 cudaError_t to_bf16(__nv_bfloat16* dst, const float* src, long n, cudaStream_t s);

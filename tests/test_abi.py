@@ -65,6 +65,8 @@ def test_create_rejects_bad_budget(lib, T, B):
     (dict(cfg=1, guidance=float("nan")), 1),
     (dict(qk_norm=2), 1),
     (dict(qk_norm=1), 7),          # QK-norm rides on the tensor-core epilogue: bf16 only
+    (dict(sampler=2), 1),
+    (dict(shift=-1.0), 1),
 ])
 def test_create_rejects_bad_arch(lib, patch, code):
     st, h, msg = _create(lib, configs.get_config("tiny"), 10, 5, **patch)

@@ -454,3 +454,46 @@ def test_qk_norm_sample_parity(name, lib):
     plain = O.sample(configs.get_config(name), synth.make_weights(configs.get_config(name)), g, inp,
                      T=T, B=B, policy=ref["mask"])
     assert float(np.max(np.abs(plain["x"] - ref["x"]))) > 10 * err
+
+
+# ---------------------------------------------------------------------------
+# samplers: UniPC (order 2 + corrector) and the time-shifted grid
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name,over", [("tiny", dict(sampler="unipc", shift=3.0)),
+                                       ("flux_small", dict(sampler="unipc")),
+                                       ("wan_small", dict(sampler="euler", shift=5.0))],
+                         ids=["tiny-unipc", "flux_small-unipc", "wan_small-euler-shift"])
+def test_sampler_variant_parity(name, over, lib):
+    cfg = configs.get_config(name, **over)
+    T, B = cfg["T"], cfg["budgets"][0]
+    inp, got, mask, log, nfe = _gpu_sample(cfg, T, B)
+    assert nfe == B and int(mask.sum()) == B
+    W, g = synth.make_weights(cfg), synth.make_gate(cfg["gate_seed"])
+    ref = O.sample(cfg, W, g, inp, T=T, B=B, drift_override=_gate_inputs(log))
+    assert list(mask) == ref["mask"]
+    rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
+    err = float(np.max(np.abs(got.astype(np.float64) - ref["x"])))
+    assert err <= TOL[cfg["dtype"]] * rms, (err, rms)
+
+
+def test_unipc_budget_T_bit_exact_and_step_api(lib):
+    """UniPC keeps its multistep history in the context: B = T equals uncached sampling
+    bit for bit, and bag_step reproduces bag_run."""
+    cfg = configs.get_config("wan_small")
+    assert cfg["sampler"] == "unipc"
+    T = 6
+    _, a, ma, _, _ = _gpu_sample(cfg, T, T)
+    _, b, mb, _, _ = _gpu_sample(cfg, T, 1, policy=bag.POLICY_FULL)
+    assert list(ma) == list(mb) == [1] * T and np.array_equal(a, b)
+    ctx = bag.create(cfg, T=T, B=3)
+    inp = synth.make_inputs(cfg)
+    x, txt, pooled = _dev_inputs(cfg, inp)
+    x0 = x.clone()
+    m_run, _, _ = ctx.run(x, txt, pooled)
+    ctx.reset()
+    xs = x0.clone()
+    for t in range(T):
+        ctx.step(xs, t, txt, pooled, xs)
+    torch.cuda.synchronize()
+    assert torch.equal(xs, x)
+    ctx.close()
