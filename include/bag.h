@@ -164,6 +164,12 @@ bag_status bag_load_gate(bag_ctx* ctx, const float* theta, int n, const float* m
  * The budget pacing of Algorithm 2 applies only to BAG_POLICY_BAG. */
 bag_status bag_set_policy(bag_ctx* ctx, int policy, const uint8_t* host_mask, float delta);
 
+/* Change the budget of later samples to B (1 <= B <= T, else EINVAL; Sec. 3.2: the target
+ * budget is set at runtime and one gate serves every budget).  The step graph is
+ * re-captured on the next run; a static evenly spaced mask is recomputed for B.  Call
+ * between samples. */
+bag_status bag_set_budget(bag_ctx* ctx, int B);
+
 /* Start a new sample: t = 0, c = 0, cache invalid, sticky device error cleared. */
 bag_status bag_reset(bag_ctx* ctx);
 

@@ -42,6 +42,7 @@ Parity pins: see tests/test_oracle_pins.py.  Every function below is pinned by a
 one closed form, invariant, special case or brute-force check there.
 """
 
+import itertools
 import math
 
 import numpy as np
@@ -516,6 +517,74 @@ def gate_logit6(f, g):
     ht = _dense32(_dense32(fz[3:], *L[2], relu=True), *L[3], relu=True)
     h = _dense32(hb + ht, *L[4], relu=True)
     return _dense32(h, *L[5], relu=False)[0]
+
+
+# ---------------------------------------------------------------------------
+# training side (Algorithm 1): Eq. 2's reference schedule and Eq. 4's loss
+# ---------------------------------------------------------------------------
+def all_masks(B, T):
+    """Every schedule with ||m||_1 = B and m_0 = 1 (Sec. 3.1), in lexicographic order of
+    the computed steps."""
+    for rest in itertools.combinations(range(1, T), B - 1):
+        m = [0] * T
+        m[0] = 1
+        for t in rest:
+            m[t] = 1
+        yield m
+
+
+def reference_by_enumeration(distance, B, T):
+    """Eq. 2 by brute force: the mask minimising distance(mask) over all matched-NFE
+    masks (the first one on ties).  Returns (mask, distance)."""
+    best, best_d = None, math.inf
+    for m in all_masks(B, T):
+        dm = distance(m)
+        if dm < best_d:
+            best, best_d = m, dm
+    return best, best_d
+
+
+def gate_forward64(g, xz):
+    """Gate logit in float64 on already z-scored inputs xz [n, k] (rows = examples):
+    the same architectures as gate_logit / gate_logit6 without fp32 rounding."""
+    xz = np.asarray(xz, np.float64)
+    relu = lambda v: np.maximum(v, 0.0)   # noqa: E731
+    if g.get("kind", "mlp3") == "mlp3":
+        return relu(xz @ np.asarray(g["w1"], np.float64).T + g["b1"]) @ np.asarray(g["w2"], np.float64) + g["b2"][0]
+    L = [(np.asarray(W, np.float64), np.asarray(b, np.float64)) for W, b in zip(g["W"], g["b"])]
+    if g["kind"] == "flux6":
+        h = xz
+        for k, (W, b) in enumerate(L):
+            h = h @ W.T + b
+            if k < len(L) - 1:
+                h = relu(h)
+        return h[:, 0]
+    hb = relu(relu(xz[:, :3] @ L[0][0].T + L[0][1]) @ L[1][0].T + L[1][1])
+    ht = relu(relu(xz[:, 3:] @ L[2][0].T + L[2][1]) @ L[3][0].T + L[3][1])
+    h = relu(np.concatenate([hb, ht], axis=1) @ L[4][0].T + L[4][1])
+    return (h @ L[5][0].T + L[5][1])[:, 0]
+
+
+def zscore_stats(X):
+    """Per-input mean and standard deviation of the training examples (Sec. 3.2: the
+    inputs are z-scored); a constant input gets sd = 1."""
+    X = np.asarray(X, np.float64)
+    mu, sd = X.mean(axis=0), X.std(axis=0)
+    return mu, np.where(sd > 0, sd, 1.0)
+
+
+def distillation_loss(g, X, y):
+    """Eq. 4 (divided by |D|), class-balanced: mean over examples of w_i BCE(sigma(z_i), y_i), z_i the gate
+    on (x_i - mu) / sd, positives weighted by the negative-to-positive count ratio
+    (App. A.2), negatives by 1.  float64."""
+    X, y = np.asarray(X, np.float64), np.asarray(y, np.float64)
+    z = gate_forward64(g, (X - g["mu"]) / g["sd"])
+    n_pos = float(y.sum())
+    w_pos = (len(y) - n_pos) / n_pos if n_pos > 0 else 1.0
+    # BCE(sigma(z), y) = softplus(z) - y z, written stably
+    sp = np.maximum(z, 0.0) + np.log1p(np.exp(-np.abs(z)))
+    per = np.where(y > 0.5, w_pos * (sp - z), sp)
+    return float(per.mean())
 
 
 def pace(gate_bit, B, T, c, t):

@@ -26,7 +26,7 @@ STATUS = {0: "BAG_OK", 1: "BAG_EINVAL", 2: "BAG_ENOMEM", 3: "BAG_ECUDA", 4: "BAG
           5: "BAG_EDEVICE_TIMEOUT", 6: "BAG_ESTATE", 7: "BAG_EUNSUPPORTED"}
 
 EXPORTS = ["bag_create", "bag_destroy", "bag_last_error", "bag_set_stream", "bag_load_gate",
-           "bag_set_policy", "bag_reset", "bag_step", "bag_run", "bag_run_host",
+           "bag_set_policy", "bag_set_budget", "bag_reset", "bag_step", "bag_run", "bag_run_host",
            "bag_get_weight", "bag_forward_block", "bag_prepare", "bag_launch_count",
            "bag_gemm_bf16", "bag_attention_bf16", "bag_ln_mod", "bag_residual_add",
            "bag_profile_run", "bag_profile_launches", "bag_rel_l1", "bag_rel_l1_noalloc"]
@@ -95,6 +95,7 @@ def load(path=None):
         "bag_set_stream": ([_P, _P], _I),
         "bag_load_gate": ([_P, _P, _I, _P, _P], _I),
         "bag_set_policy": ([_P, _I, _P, ctypes.c_float], _I),
+        "bag_set_budget": ([_P, _I], _I),
         "bag_reset": ([_P], _I),
         "bag_step": ([_P, _P, _I, ctypes.POINTER(Cond), _P, _P], _I),
         "bag_run": ([_P, _P, ctypes.POINTER(Cond), ctypes.POINTER(Stats)], _I),
@@ -202,6 +203,11 @@ class Context:
         m = None if mask is None else np.ascontiguousarray(mask, np.uint8)
         self._chk(self.lib.bag_set_policy(self.h, policy, None if m is None else m.ctypes.data,
                                           float(delta)))
+
+    def set_budget(self, B):
+        """Budget of later samples (the step graph is re-captured on the next run)."""
+        self._chk(self.lib.bag_set_budget(self.h, int(B)))
+        self.B = int(B)
 
     def reset(self):
         self._chk(self.lib.bag_reset(self.h))

@@ -1710,9 +1710,20 @@ bag_status bag_set_policy(bag_ctx* ctx, int policy, const uint8_t* host_mask, fl
     CK(cudaStreamSynchronize(ctx->stream));
   }
   if (policy == BAG_POLICY_THRESHOLD && !(delta == delta)) return fail(ctx, BAG_EINVAL, "delta is NaN");
+  // policy and delta are kernel arguments of the captured gate launch; a new mask is
+  // device data the same graph reads
+  if (policy != ctx->policy || delta != ctx->delta) destroy_graph(ctx);
   ctx->policy = policy;
   ctx->delta = delta;
-  destroy_graph(ctx);  // policy and delta are kernel arguments of the captured gate launch
+  return BAG_OK;
+}
+
+bag_status bag_set_budget(bag_ctx* ctx, int B) {
+  if (!ctx) return BAG_EINVAL;
+  if (B < 1 || B > ctx->T) return fail(ctx, BAG_EINVAL, "need 1 <= B <= T");
+  ctx->B = B;
+  destroy_graph(ctx);  // B is a kernel argument of the captured gate launch
+  if (ctx->policy == BAG_POLICY_STATIC_UNIFORM) return bag_set_policy(ctx, ctx->policy, nullptr, ctx->delta);
   return BAG_OK;
 }
 

@@ -85,6 +85,7 @@ def test_null_arguments(lib):
     h = ctypes.c_void_p()
     assert lib.bag_create(None, 10, 5, ctypes.byref(h)) == 1
     assert lib.bag_reset(None) == 1
+    assert lib.bag_set_budget(None, 3) == 1
     assert lib.bag_run(None, None, None, None) == 1
     lib.bag_destroy(None)
 

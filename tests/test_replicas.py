@@ -33,7 +33,7 @@ def _worker(rank, world, port, out):
 @pytest.mark.parametrize("world", [2])
 def test_two_gloo_replicas(world):
     port = 29500 + (os.getpid() % 2000)
-    with mp.Manager() as m:
+    with mp.get_context("spawn").Manager() as m:
         out = m.dict()
         mp.spawn(_worker, args=(world, port, out), nprocs=world, join=True)
         res = dict(out)
