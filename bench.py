@@ -166,6 +166,7 @@ KERNEL_NAMES = {"gemm": "gemm_tc_kernel", "attention": "attn_tc_kernel",
                 "norm": "ln_mod_kernel", "signal": "ln_mod_kernel (signal)",
                 "gate": "gate_kernel", "cache": "cache_refresh/reuse_kernel"}
 KERNEL_SOURCES = {"gemm_tc_kernel": ["gemm.cu", "epilogue.cuh", "common.cuh"],
+                  "gemm_pair_kernel": ["gemm.cu", "epilogue.cuh", "common.cuh"],
                   "attn_tc_kernel": ["attn_tc.cu", "common.cuh"]}
 
 
@@ -197,15 +198,17 @@ def dominant_roofline(recs, peaks, peak_src, cfg_name, f32=False):
     configurations run on the CUDA cores; their bound is the fp32 FMA rate."""
     groups = {}
     for r in recs:
-        key = (r["kind"], r["m"], r["n"], r["k"])
+        key = (r["kind"], r["m"], r["n"], r["k"], r.get("variant", 0))
         g = groups.setdefault(key, {"launches": 0, "ms": 0.0, "flops": 0.0, "bytes": 0.0})
         g["launches"] += 1
         g["ms"] += r["ms"]
         g["flops"] += r["flops"]
         g["bytes"] += r["bytes"]
-    kind, m, n, k = max(groups, key=lambda q: groups[q]["ms"])
-    g = groups[(kind, m, n, k)]
+    kind, m, n, k, variant = max(groups, key=lambda q: groups[q]["ms"])
+    g = groups[(kind, m, n, k, variant)]
     name = KERNEL_NAMES[kind]
+    if kind == "gemm" and variant == 1:
+        name = "gemm_pair_kernel"
     if f32 and kind in ("gemm", "attention"):
         name = {"gemm": "gemm_simt_kernel", "attention": "attn_simt_kernel"}[kind]
     avg_ms = g["ms"] / g["launches"]

@@ -237,12 +237,14 @@ bag_status bag_profile_run(bag_ctx* ctx, float* x_inout, const bag_cond* cond, b
                            bag_prof_entry* out);
 
 /* Per-launch records of the last bag_profile_run: kind (BAG_PROF_*), shape (GEMM: M, N,
- * K; attention: n_q, n_k, heads; 0 otherwise), event time, algorithmic flops and bytes.
+ * K; attention: n_q, n_k, heads; 0 otherwise), event time, algorithmic flops and bytes,
+ * and the kernel variant (GEMM: 1 = CTA-pair kernel, 0 = single-CTA kernel; else 0).
  * *n receives the number of records; up to max are copied to out (host; may be null). */
 typedef struct {
   int kind, m, n, k;
   float ms;
   double flops, bytes;
+  int variant;
 } bag_prof_launch;
 bag_status bag_profile_launches(bag_ctx* ctx, bag_prof_launch* out, long max, long* n);
 

@@ -64,7 +64,7 @@ class ProfEntry(ctypes.Structure):
 class ProfLaunch(ctypes.Structure):
     _fields_ = [("kind", ctypes.c_int), ("m", ctypes.c_int), ("n", ctypes.c_int),
                 ("k", ctypes.c_int), ("ms", ctypes.c_float), ("flops", ctypes.c_double),
-                ("bytes", ctypes.c_double)]
+                ("bytes", ctypes.c_double), ("variant", ctypes.c_int)]
 
 
 class Stats(ctypes.Structure):
@@ -252,7 +252,7 @@ class Context:
         arr = (ProfLaunch * max(1, n.value))()
         self._chk(self.lib.bag_profile_launches(self.h, arr, n.value, ctypes.byref(n)))
         return [dict(kind=PROF_KINDS[r.kind], m=r.m, n=r.n, k=r.k, ms=r.ms, flops=r.flops,
-                     bytes=r.bytes) for r in arr[:n.value]]
+                     bytes=r.bytes, variant=r.variant) for r in arr[:n.value]]
 
     def run_host(self, x, txt, pooled, txt_u=None, pooled_u=None):
         """All T steps with host numpy buffers (x updated in place); returns (mask, log, nfe)."""

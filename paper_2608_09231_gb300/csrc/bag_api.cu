@@ -169,6 +169,7 @@ struct bag_ctx {
     double flops, bytes;
     int e0, e1;
     int m, n, k;
+    int variant;
   };
   std::vector<ProfRec> prof;
   std::vector<cudaEvent_t> ev_pool;
@@ -698,11 +699,13 @@ struct Enq {
   cudaStream_t s;
   long* count;
   cudaError_t e = cudaSuccess;
-  int pk = -1, pe0 = -1, pm = 0, pn = 0, pkk = 0;
+  int pk = -1, pe0 = -1, pm = 0, pn = 0, pkk = 0, pv = 0;
   double pf = 0, pb = 0;
-  // announce the next launch (kind, algorithmic flops and bytes, shape) for profiling
-  void pre(int kind, double flops, double bytes, int m = 0, int n = 0, int k = 0) {
+  // announce the next launch (kind, algorithmic flops and bytes, shape, kernel variant)
+  // for profiling
+  void pre(int kind, double flops, double bytes, int m = 0, int n = 0, int k = 0, int variant = 0) {
     if (!ctx->profiling) return;
+    pv = variant;
     pe0 = prof_event(ctx);
     if (pe0 < 0) return;
     cudaEventRecord(ctx->ev_pool[pe0], s);
@@ -720,7 +723,7 @@ struct Enq {
       const int pe1 = prof_event(ctx);
       if (pe1 >= 0) {
         cudaEventRecord(ctx->ev_pool[pe1], s);
-        ctx->prof.push_back({pk, pf, pb, pe0, pe1, pm, pn, pkk});
+        ctx->prof.push_back({pk, pf, pb, pe0, pe1, pm, pn, pkk, pv});
       }
       pk = -1;
     }
@@ -746,7 +749,8 @@ static void enq_gemm(Enq& q, const void* A, long lda, const Tensor& W, long ldw,
     double out = (double)M * N * 4;
     if (e.kind == EPI_GATED_RES || e.kind == EPI_RES_ADD) out = (double)M * N * 8;
     else if (e.kind == EPI_QKV || e.kind == EPI_GELU) out = (double)M * N * es;
-    q.pre(BAG_PROF_GEMM, 2.0 * M * N * K, ((double)M + N) * K * es + out, M, N, K);
+    q.pre(BAG_PROF_GEMM, 2.0 * M * N * K, ((double)M + N) * K * es + out, M, N, K,
+          q.ctx->act_bf16 ? gemm_uses_pair(M, 0, N) : 0);
   }
   q.chk(gemm(A, lda, W.p, ldw, M, N, K, q.ctx->act_bf16, e, q.ctx->st ? &q.ctx->st->err : nullptr, q.s));
 }
@@ -766,7 +770,7 @@ static void enq_gemm2(Enq& q, const void* A0, long lda0, const Tensor& W0, long 
   if (e0.kind == EPI_GATED_RES || e0.kind == EPI_RES_ADD) out = (double)(M0 + M1) * N * 8;
   else if (e0.kind == EPI_QKV || e0.kind == EPI_GELU) out = (double)(M0 + M1) * N * es;
   q.pre(BAG_PROF_GEMM, 2.0 * (M0 + M1) * N * K, ((double)M0 + M1 + 2.0 * N) * K * es + out,
-        M0 + M1, N, K);
+        M0 + M1, N, K, gemm_uses_pair(M0, M1, N));
   q.chk(gemm2(A0, lda0, W0.p, ldw0, M0, e0, A1, lda1, W1.p, ldw1, M1, e1, N, K,
               q.ctx->st ? &q.ctx->st->err : nullptr, q.s));
 }
@@ -1160,7 +1164,8 @@ static bag_status enq_prepare(bag_ctx* ctx, const bag_cond* cond) {
   auto gemm_f32_act = [&](const float* act, int K, const Tensor& W, int N, const Epi& e) {
     if (bf) {
       q.chk(split_bf16(ctx->splitbuf, act, ctx->T, K, s));
-      q.pre(BAG_PROF_GEMM, 4.0 * ctx->T * N * K, (double)N * K * 2, ctx->T, N, 2 * K);
+      q.pre(BAG_PROF_GEMM, 4.0 * ctx->T * N * K, (double)N * K * 2, ctx->T, N, 2 * K,
+            gemm_uses_pair(ctx->T, 0, N));
       q.chk(gemm(ctx->splitbuf, 2L * K, W.p, K, ctx->T, N, K, 1, e, &ctx->st->err, s, 0, 1));
     } else {
       enq_gemm(q, act, K, W, K, ctx->T, N, K, e);
@@ -1808,7 +1813,7 @@ bag_status bag_profile_launches(bag_ctx* ctx, bag_prof_launch* out, long max, lo
     const auto& r = ctx->prof[i];
     float ms = 0.f;
     cudaEventElapsedTime(&ms, ctx->ev_pool[r.e0], ctx->ev_pool[r.e1]);
-    out[i] = bag_prof_launch{r.kind, r.m, r.n, r.k, ms, r.flops, r.bytes};
+    out[i] = bag_prof_launch{r.kind, r.m, r.n, r.k, ms, r.flops, r.bytes, r.variant};
   }
   return BAG_OK;
 }

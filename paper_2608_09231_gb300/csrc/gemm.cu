@@ -125,6 +125,51 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
 // ---------------------------------------------------------------------------
 constexpr int TC_BM = 128, TC_BK = 64;
 
+// One thread's row of a BN-column accumulator in TMEM (lane base already in tb) through
+// the epilogue, columns col0 .. col0 + BN - 1.
+template <int BN>
+BAG_DEV void drain_accumulator(const Epi& e, int t, int row, int col0, uint32_t tb) {
+  if (e.qn_q) {
+    // QK-norm: the tile holds whole heads (BN a multiple of dh, checked at launch); a
+    // first pass over each q / k head takes its sum of squares (bias included), the
+    // second applies the epilogue with 1 / RMS.  The TMEM loads are warp-wide, so every
+    // lane takes them whatever its row.
+    const int dh = e.dh;
+#pragma unroll 1
+    for (int h0 = 0; h0 < BN; h0 += dh) {
+      const int col = col0 + h0;
+      float rs = 1.f;
+      if ((col + e.col_base) / e.d < 2 && col < e.N) {
+        float ss = 0.f;
+#pragma unroll 1
+        for (int c = 0; c < dh; c += 32) {
+          float v[32];
+          tmem_ld32(tb + (uint32_t)(h0 + c), v);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const float x = v[j] + (e.bias ? __ldg(e.bias + col + c + j) : 0.f);
+            ss = fmaf(x, x, ss);
+          }
+        }
+        rs = rsqrtf(ss / (float)dh + 1e-6f);
+      }
+#pragma unroll 1
+      for (int c = 0; c < dh; c += 32) {
+        float v[32];
+        tmem_ld32(tb + (uint32_t)(h0 + c), v);
+        epi_apply<32>(e, t, row, col + c, v, rs);
+      }
+    }
+  } else {
+#pragma unroll 1
+    for (int c = 0; c < BN / 32; ++c) {
+      float v[32];
+      tmem_ld32(tb + (uint32_t)(c * 32), v);
+      epi_apply<32>(e, t, row, col0 + c * 32, v);
+    }
+  }
+}
+
 template <int BN>
 struct TcCfg {
   static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
@@ -311,45 +356,7 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_after();
       const int row = mt * TC_BM + q * 32 + lane;
       const uint32_t tb = tmem_base + (uint32_t)(acc * BN) + ((uint32_t)(q * 32) << 16);
-      if (e.qn_q) {
-        // QK-norm: the tile holds whole heads (BN a multiple of dh, checked at launch);
-        // a first pass over each q / k head takes its sum of squares (bias included),
-        // the second applies the epilogue with 1 / RMS.  The TMEM loads are warp-wide,
-        // so every lane takes them whatever its row.
-        const int dh = e.dh;
-#pragma unroll 1
-        for (int h0 = 0; h0 < BN; h0 += dh) {
-          const int col = nt * BN + h0;
-          float rs = 1.f;
-          if ((col + e.col_base) / e.d < 2 && col < e.N) {
-            float ss = 0.f;
-#pragma unroll 1
-            for (int c = 0; c < dh; c += 32) {
-              float v[32];
-              tmem_ld32(tb + (uint32_t)(h0 + c), v);
-#pragma unroll
-              for (int j = 0; j < 32; ++j) {
-                const float x = v[j] + (e.bias ? __ldg(e.bias + col + c + j) : 0.f);
-                ss = fmaf(x, x, ss);
-              }
-            }
-            rs = rsqrtf(ss / (float)dh + 1e-6f);
-          }
-#pragma unroll 1
-          for (int c = 0; c < dh; c += 32) {
-            float v[32];
-            tmem_ld32(tb + (uint32_t)(h0 + c), v);
-            epi_apply<32>(e, t, row, col + c, v, rs);
-          }
-        }
-      } else {
-#pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
-          float v[32];
-          tmem_ld32(tb + (uint32_t)(c * 32), v);
-          epi_apply<32>(e, t, row, nt * BN + c * 32, v);
-        }
-      }
+      drain_accumulator<BN>(e, t, row, nt * BN, tb);
       tc_fence_before();
       mbar_arrive(tempty + acc);
       acc ^= 1;
@@ -390,6 +397,250 @@ static cudaError_t launch_tc(const void* A0, long lda0, const void* W0, long ldw
   return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------
+// CTA-pair GEMM: clusters of two CTAs compute 256 x 256 tiles with cta_group::2 MMAs
+// (M = 256, N = 256, K = 16 per instruction).  Each CTA stages its own 128 rows of A
+// and 128 rows of W per k-block (32 KB instead of the single-CTA 128 x 256 tile's
+// 48 KB), so every SM moves a third less shared-memory operand data per MMA cycle, the
+// limit of the single-CTA kernel.  Roles as in gemm_tc_kernel: warp 0 of each CTA loads
+// its halves (completion signalled on the even CTA's barrier), warp 1 of the even CTA
+// issues the MMAs and multicasts their completion to both CTAs, warps 2..5 of each CTA
+// drain its 128 accumulator rows.
+// ---------------------------------------------------------------------------
+constexpr int PR_BM = 256, PR_BN = 256, PR_STAGES = 6;
+constexpr int PR_HALF_BYTES = 128 * TC_BK * 2;  // one CTA's A or W half-tile per k-block
+constexpr int PR_STAGE_BYTES = 2 * PR_HALF_BYTES;
+constexpr int PR_TMEM_COLS = 2 * PR_BN;         // double-buffered accumulator
+constexpr int PR_SMEM = PR_STAGES * PR_STAGE_BYTES + 1024 + 256;
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
+    gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
+                     const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
+                     const __grid_constant__ Epi e0, const __grid_constant__ Epi e1, int M0, int M1,
+                     int N, int K, int a_split, int* err) {
+  // both CTAs of a pair see the same flag, so they leave together
+  if (epi_skip(e0.st, e0.flag_want)) return;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + PR_STAGES * PR_HALF_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + PR_STAGES * PR_STAGE_BYTES);
+  uint64_t* empty = full + PR_STAGES;
+  uint64_t* tfull = empty + PR_STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const uint32_t rank = cluster_ctarank();
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+  const int num_m0 = (M0 + PR_BM - 1) / PR_BM, num_m1 = (M1 + PR_BM - 1) / PR_BM, num_n = N / PR_BN;
+  const int tiles0 = num_m0 * num_n;
+  auto decode = [&](int tile, int& pb, int& mt, int& nt) {
+    if (tile < tiles0) {
+      pb = 0;
+      mt = tile % num_m0;
+      nt = tile / num_m0;
+    } else {
+      const int l = tile - tiles0;
+      pb = 1;
+      mt = l % num_m1;
+      nt = l / num_m1;
+    }
+  };
+  const int tiles = tiles0 + num_m1 * num_n, kit = (a_split ? 2 : 1) * (K / TC_BK);
+  const int t = epi_step(e0);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < PR_STAGES; ++s) {
+      mbar_init(full + s, 1);   // even CTA: its producer's expect_tx; both CTAs' bytes
+      mbar_init(empty + s, 1);  // both CTAs: one multicast commit per consumed stage
+    }
+    mbar_init(tfull, 1);
+    mbar_init(tfull + 1, 1);
+    mbar_init(tempty, 256);     // even CTA: every epilogue thread of both CTAs
+    mbar_init(tempty + 1, 256);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA0);
+    tma_prefetch_desc(&tmB0);
+    if (M1 > 0) {
+      tma_prefetch_desc(&tmA1);
+      tma_prefetch_desc(&tmB1);
+    }
+  }
+  __syncwarp();
+  if (warp == 1) {
+    tmem_alloc_pair(tmem_slot, PR_TMEM_COLS);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncwarp();
+  cluster_sync_all();  // barriers of both CTAs initialised, tensor memory allocated
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer (both CTAs: their own halves) ----------------
+      int s = 0;
+      uint32_t ph = 0;
+      long issued = 0;
+      bool ok = true;
+      for (int tile = pair; tile < tiles && ok; tile += npairs) {
+        int pb, mt, nt;
+        decode(tile, pb, mt, nt);
+        const CUtensorMap* tmA = pb ? &tmA1 : &tmA0;
+        const CUtensorMap* tmB = pb ? &tmB1 : &tmB0;
+        for (int kb = 0; kb < kit; ++kb) {
+          if (!mbar_wait(empty + s, ph ^ 1, abort_flag)) {
+            ok = false;
+            break;
+          }
+          if (rank == 0) mbar_arrive_expect_tx(full + s, 2 * PR_STAGE_BYTES);
+          const uint32_t fb = mapa_shared(smem_u32(full + s), 0);
+          const int ka = a_split ? (kb & 1) * K + (kb >> 1) * TC_BK : kb * TC_BK;
+          const int kw = a_split ? (kb >> 1) * TC_BK : kb * TC_BK;
+          tma_load_2d_pair(sA + s * PR_HALF_BYTES, tmA, ka, mt * PR_BM + (int)rank * 128, fb);
+          tma_load_2d_pair(sB + s * PR_HALF_BYTES, tmB, kw, nt * PR_BN + (int)rank * 128, fb);
+          ++issued;
+          if (++s == PR_STAGES) {
+            s = 0;
+            ph ^= 1;
+          }
+        }
+      }
+      if (!ok && rank == 0) {
+        // drain (bounded): both CTAs' copies in flight complete on this CTA's barriers
+        const uint64_t t0 = global_ns();
+        for (int i = 0; i < PR_STAGES && i < issued; ++i) {
+          if (--s < 0) {
+            s = PR_STAGES - 1;
+            ph ^= 1;
+          }
+          while (!mbar_try_wait(full + s, ph) && global_ns() - t0 < kWaitLimitNs) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      // ---------------- MMA issuer (even CTA) ----------------
+      constexpr uint32_t idesc = idesc_bf16_f32(PR_BM, PR_BN);
+      int s = 0;
+      uint32_t ph = 0;
+      int acc = 0;
+      uint32_t aph = 0;
+      bool ok = true;
+      for (int tile = pair; tile < tiles && ok; tile += npairs) {
+        if (!mbar_wait(tempty + acc, aph ^ 1, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t dt = tmem_base + (uint32_t)(acc * PR_BN);
+        for (int kb = 0; kb < kit; ++kb) {
+          if (!mbar_wait(full + s, ph, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + s * PR_HALF_BYTES);
+          const uint32_t b0 = smem_u32(sB + s * PR_HALF_BYTES);
+#pragma unroll
+          for (int k = 0; k < TC_BK / 16; ++k)
+            mma_bf16_pair(dt, sw128_desc(a0 + k * 32), sw128_desc(b0 + k * 32), idesc,
+                          (kb | k) != 0 ? 1u : 0u);
+          mma_commit_pair(empty + s, 3);
+          if (++s == PR_STAGES) {
+            s = 0;
+            ph ^= 1;
+          }
+        }
+        if (!ok) break;
+        mma_commit_pair(tfull + acc, 3);
+        acc ^= 1;
+        if (acc == 0) aph ^= 1;
+      }
+      // every issued MMA has finished before tensor memory is released
+      mma_commit_pair(drain, 1);
+      const uint64_t t0 = global_ns();
+      while (!mbar_try_wait(drain, 0) && global_ns() - t0 < kWaitLimitNs) {
+      }
+    }
+  } else {
+    // ---------------- epilogue (both CTAs: their 128 rows of each tile) ----------------
+    const int q = warp & 3;
+    int acc = 0;
+    uint32_t aph = 0;
+    const uint32_t te_remote = mapa_shared(smem_u32(tempty), 0);
+    for (int tile = pair; tile < tiles; tile += npairs) {
+      int pb, mt, nt;
+      decode(tile, pb, mt, nt);
+      const Epi& e = pb ? e1 : e0;
+      bool ok = mbar_wait(tfull + acc, aph, abort_flag);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      tc_fence_after();
+      const int row = mt * PR_BM + (int)rank * 128 + q * 32 + lane;
+      const uint32_t tb = tmem_base + (uint32_t)(acc * PR_BN) + ((uint32_t)(q * 32) << 16);
+      drain_accumulator<PR_BN>(e, t, row, nt * PR_BN, tb);
+      tc_fence_before();
+      if (rank == 0)
+        mbar_arrive(tempty + acc);
+      else
+        mbar_arrive_remote(te_remote + (uint32_t)(acc * sizeof(uint64_t)));
+      acc ^= 1;
+      if (acc == 0) aph ^= 1;
+    }
+  }
+  tc_fence_before();
+  __syncwarp();
+  cluster_sync_all();  // no CTA of the pair still uses the pair's tensor memory
+  if (threadIdx.x == 0 && *abort_flag && err) atomicOr(err, 1);
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, PR_TMEM_COLS);
+  }
+}
+
+// Tiles of the pair kernel for a launch of one or two problems; it is used when N is a
+// multiple of 256 and there are at least as many 256 x 256 tiles as CTA pairs.
+static int pair_tiles(int M0, int M1, int N) {
+  return ((M0 + PR_BM - 1) / PR_BM + (M1 + PR_BM - 1) / PR_BM) * (N / PR_BN);
+}
+
+static cudaError_t launch_pair(const void* A0, long lda0, const void* W0, long ldw0, int M0,
+                               const Epi& e0, const void* A1, long lda1, const void* W1, long ldw1,
+                               int M1, const Epi& e1, int N, int K, int* err, cudaStream_t s,
+                               int a_split) {
+  const uint64_t ka = (uint64_t)K * (a_split ? 2 : 1);
+  CUtensorMap ta0, tb0, ta1, tb1;
+  if (encode_tmap_2d_bf16(&ta0, A0, ka, (uint64_t)M0, (uint64_t)lda0 * 2, TC_BK, 128) ||
+      encode_tmap_2d_bf16(&tb0, W0, (uint64_t)K, (uint64_t)N, (uint64_t)ldw0 * 2, TC_BK, 128))
+    return cudaErrorInvalidValue;
+  if (M1 > 0) {
+    if (encode_tmap_2d_bf16(&ta1, A1, ka, (uint64_t)M1, (uint64_t)lda1 * 2, TC_BK, 128) ||
+        encode_tmap_2d_bf16(&tb1, W1, (uint64_t)K, (uint64_t)N, (uint64_t)ldw1 * 2, TC_BK, 128))
+      return cudaErrorInvalidValue;
+  } else {
+    ta1 = ta0;
+    tb1 = tb0;
+  }
+  const int pairs = std::min(pair_tiles(M0, M1, N), num_sms() / 2);
+  gemm_pair_kernel<<<2 * pairs, 192, PR_SMEM, s>>>(ta0, tb0, ta1, tb1, e0, e1, M0, M1, N, K, a_split,
+                                                   err);
+  return cudaGetLastError();
+}
+
+int gemm_uses_pair(int M0, int M1, int N) {
+  return N % PR_BN == 0 && num_sms() >= 2 && pair_tiles(M0, M1, N) >= num_sms() / 2;
+}
+
 cudaError_t attention_tc_init();
 
 cudaError_t kernels_init() {
@@ -401,6 +652,8 @@ cudaError_t kernels_init() {
   if (r == cudaSuccess)
     r = cudaFuncSetAttribute(gemm_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              TcCfg<64>::SMEM);
+  if (r == cudaSuccess)
+    r = cudaFuncSetAttribute(gemm_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, PR_SMEM);
   if (r == cudaSuccess) r = attention_tc_init();
   num_sms();
   return r;
@@ -430,6 +683,9 @@ static cudaError_t gemm_tc2(const void* A0, long lda0, const void* W0, long ldw0
   const bool qkn = e0.qn_q || (M1 > 0 && e1.qn_q);
   const int min_bn = qkn ? e0.dh : 64;
   if (qkn && (e0.dh % 32 || (M1 > 0 && e1.dh != e0.dh) || min_bn > 256)) return cudaErrorNotSupported;
+  if (gemm_uses_pair(M0, M1 > 0 ? M1 : 0, N))
+    return launch_pair(A0, lda0, W0, ldw0, M0, e0, A1, lda1, W1, ldw1, M1 > 0 ? M1 : 0, e1, N, K, err, s,
+                       a_split);
   if (N % 256 == 0 && (mt * (N / 256) >= ns || min_bn > 128))
     return launch_tc<256>(A0, lda0, W0, ldw0, M0, e0, A1, lda1, W1, ldw1, M1, e1, N, K, err, s, a_split);
   if (min_bn > 128) return cudaErrorNotSupported;

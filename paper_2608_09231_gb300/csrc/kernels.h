@@ -116,6 +116,8 @@ cudaError_t gemm(const void* A, long lda, const void* W, long ldw, int M, int N,
 // dst [rows, 2*cols] bf16 = [bf16(x) | bf16(x - bf16(x))] of src fp32 [rows, cols]
 cudaError_t split_bf16(__nv_bfloat16* dst, const float* src, long rows, long cols, cudaStream_t s);
 int gemm_tc_supported(int M, int N, int K, long lda, long ldw);
+// 1 when a bf16 launch of these shapes runs on the CTA-pair kernel (gemm_pair_kernel)
+int gemm_uses_pair(int M0, int M1, int N);
 // Two bf16 problems with the same N and K in one tensor-core launch (e.g. the image and
 // text streams of a double-stream block); M1 may be 0.
 cudaError_t gemm2(const void* A0, long lda0, const void* W0, long ldw0, int M0, const Epi& epi0,

@@ -169,8 +169,11 @@ def _bf16_tensor(seed, shape, std=1.0):
     return v, torch.from_numpy(v).cuda().to(torch.bfloat16)
 
 
+# (4096, 3072, 3072), (1000, 19456, 192) and (4100, 4864, 320) have enough 256 x 256
+# tiles for the CTA-pair kernel (the last two with a ragged final row tile)
 @pytest.mark.parametrize("M,N,K", [(300, 256, 128), (129, 64, 64), (1000, 384, 512),
-                                   (77, 512, 256), (4096, 3072, 3072), (50, 1024, 320)])
+                                   (77, 512, 256), (4096, 3072, 3072), (50, 1024, 320),
+                                   (1000, 19456, 192), (4100, 4864, 320)])
 @pytest.mark.parametrize("simt", [0, 1])
 def test_gemm_bf16_against_fp64(M, N, K, simt, lib):
     ctx = bag.create("tiny", T=2, B=1)
@@ -181,7 +184,7 @@ def test_gemm_bf16_against_fp64(M, N, K, simt, lib):
     C = torch.zeros((M, N), dtype=torch.float32, device="cuda")
     ctx.gemm_bf16(A, Wt, bias, C, M, N, K, 0, simt)
     torch.cuda.synchronize()
-    rows = np.arange(M) if M <= 1100 else np.r_[0:64, M - 64:M, 1000:1010]
+    rows = np.arange(M) if M * N <= 1100 * 4096 else np.r_[0:64, M - 64:M, 500:510]
     ref = a[rows].astype(np.float64) @ w.T.astype(np.float64) + b
     bound = 4 * K * 2.0 ** -24 * (np.abs(a[rows]).astype(np.float64) @ np.abs(w).T) + 1e-7
     got = C.cpu().numpy()[rows]
@@ -189,9 +192,9 @@ def test_gemm_bf16_against_fp64(M, N, K, simt, lib):
     ctx.close()
 
 
-def test_gemm_gelu_epilogue(lib):
+@pytest.mark.parametrize("M,N,K", [(257, 128, 192), (700, 19456, 128)])
+def test_gemm_gelu_epilogue(M, N, K, lib):
     ctx = bag.create("tiny", T=2, B=1)
-    M, N, K = 257, 128, 192
     a, A = _bf16_tensor(4, (M, K))
     w, Wt = _bf16_tensor(5, (N, K), 0.1)
     C = torch.zeros((M, N), dtype=torch.float32, device="cuda")
