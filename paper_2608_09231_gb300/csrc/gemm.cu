@@ -125,6 +125,33 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
 // ---------------------------------------------------------------------------
 constexpr int TC_BM = 128, TC_BK = 64;
 
+// Tile order within one problem: groups of G row tiles, each group visiting every
+// column tile with the row tile varying fastest.  A wave of tiles then shares at most G
+// row tiles of A (which stay in L2 while the group walks the columns) instead of
+// streaming all of A once per column tile; G comes from the L2 share one group's rows
+// may take (tile_group_rows).
+BAG_DEV void raster(int l, int num_m, int num_n, int G, int& mt, int& nt) {
+  const int per_group = G * num_n;
+  const int g = l / per_group;
+  const int idx = l - g * per_group;
+  const int gm = min(G, num_m - g * G);
+  mt = g * G + idx % gm;
+  nt = idx / gm;
+}
+
+#ifndef BAG_TILE_GROUP_L2_MB
+#define BAG_TILE_GROUP_L2_MB 40
+#endif
+// Row tiles per group: as many BM-row slices of A (K bf16 columns, twice as many for a
+// split A) as fit in the L2 share, at least 1, at most all of them.
+static int tile_group_rows(int M, int BM, int K, int a_split) {
+  const int num_m = (M + BM - 1) / BM;
+  if (num_m <= 0) return 1;
+  const double slice = (double)BM * K * 2.0 * (a_split ? 2 : 1);
+  const int g = (int)((double)BAG_TILE_GROUP_L2_MB * 1048576.0 / slice);
+  return std::max(1, std::min(num_m, g));
+}
+
 // One thread's row of a BN-column accumulator in TMEM (lane base already in tb) through
 // the epilogue, columns col0 .. col0 + BN - 1.
 template <int BN>
@@ -185,7 +212,7 @@ __global__ void __launch_bounds__(192, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
                    const __grid_constant__ Epi e0, const __grid_constant__ Epi e1, int M0, int M1,
-                   int N, int K, int a_split, int* err) {
+                   int N, int K, int a_split, int g0, int g1, int* err) {
   // Two independent problems with the same N and K may share one launch (problem 1 has
   // M1 rows, possibly 0): their tiles form one list, problem 0's first, so a small
   // problem fills the SMs the large one leaves idle in its last wave.
@@ -210,13 +237,10 @@ __global__ void __launch_bounds__(192, 1)
   auto decode = [&](int tile, int& pb, int& mt, int& nt) {
     if (tile < tiles0) {
       pb = 0;
-      mt = tile % num_m0;
-      nt = tile / num_m0;
+      raster(tile, num_m0, num_n, g0, mt, nt);
     } else {
-      const int l = tile - tiles0;
       pb = 1;
-      mt = l % num_m1;
-      nt = l / num_m1;
+      raster(tile - tiles0, num_m1, num_n, g1, mt, nt);
     }
   };
   // a_split: A holds [hi | lo] bf16 halves of an fp32 activation ([M, 2K]); the K loop
@@ -392,8 +416,9 @@ static cudaError_t launch_tc(const void* A0, long lda0, const void* W0, long ldw
   }
   const int tiles = ((M0 + TC_BM - 1) / TC_BM + (M1 + TC_BM - 1) / TC_BM) * (N / BN);
   const int grid = std::min(tiles, num_sms());
-  gemm_tc_kernel<BN><<<grid, 192, C::SMEM, s>>>(ta0, tb0, ta1, tb1, e0, e1, M0, M1, N, K,
-                                                a_split, err);
+  gemm_tc_kernel<BN><<<grid, 192, C::SMEM, s>>>(ta0, tb0, ta1, tb1, e0, e1, M0, M1, N, K, a_split,
+                                                tile_group_rows(M0, TC_BM, K, a_split),
+                                                tile_group_rows(M1, TC_BM, K, a_split), err);
   return cudaGetLastError();
 }
 
@@ -417,7 +442,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
     gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
                      const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
                      const __grid_constant__ Epi e0, const __grid_constant__ Epi e1, int M0, int M1,
-                     int N, int K, int a_split, int* err) {
+                     int N, int K, int a_split, int g0, int g1, int* err) {
   // both CTAs of a pair see the same flag, so they leave together
   if (epi_skip(e0.st, e0.flag_want)) return;
   extern __shared__ uint8_t smem_raw[];
@@ -441,13 +466,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
   auto decode = [&](int tile, int& pb, int& mt, int& nt) {
     if (tile < tiles0) {
       pb = 0;
-      mt = tile % num_m0;
-      nt = tile / num_m0;
+      raster(tile, num_m0, num_n, g0, mt, nt);
     } else {
-      const int l = tile - tiles0;
       pb = 1;
-      mt = l % num_m1;
-      nt = l / num_m1;
+      raster(tile - tiles0, num_m1, num_n, g1, mt, nt);
     }
   };
   const int tiles = tiles0 + num_m1 * num_n, kit = (a_split ? 2 : 1) * (K / TC_BK);
@@ -633,7 +655,8 @@ static cudaError_t launch_pair(const void* A0, long lda0, const void* W0, long l
   }
   const int pairs = std::min(pair_tiles(M0, M1, N), num_sms() / 2);
   gemm_pair_kernel<<<2 * pairs, 192, PR_SMEM, s>>>(ta0, tb0, ta1, tb1, e0, e1, M0, M1, N, K, a_split,
-                                                   err);
+                                                   tile_group_rows(M0, PR_BM, K, a_split),
+                                                   tile_group_rows(M1, PR_BM, K, a_split), err);
   return cudaGetLastError();
 }
 
