@@ -53,6 +53,28 @@ BAG_DEV float ex2(float x) {
   return y;
 }
 
+// Three-input maximum and packed two-lane fp32 FMA / add (one instruction each for two
+// elements of the S row, halving the softmax's issue slots for these steps).
+BAG_DEV float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+BAG_DEV void fma2(float& d0, float& d1, float a0, float a1, float b, float c) {
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %4};\n\tmov.b64 rc, {%5, %5};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "f"(b), "f"(c));
+}
+BAG_DEV void add2(float& d0, float& d1, float a0, float a1) {
+  asm("{\n\t.reg .b64 ra, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rd, {%0, %1};\n\t"
+      "add.rn.f32x2 rd, rd, ra;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "+f"(d0), "+f"(d1)
+      : "f"(a0), "f"(a1));
+}
+
 // 32 consecutive 32-bit TMEM columns of this thread's lane, without the wait (the caller
 // issues tcgen05.wait::ld once for several loads)
 BAG_DEV void tmem_ld32_nowait(uint32_t taddr, uint32_t* r) {
@@ -278,9 +300,16 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         for (int i = 0; i < AT_N; ++i)
           if (i >= kvalid) r[i] = __float_as_uint(-INFINITY);
       }
-      float mx = __uint_as_float(r[0]);
+      // row maximum: four independent chains of three-input maxima
+      float mq[4];
 #pragma unroll
-      for (int i = 1; i < AT_N; ++i) mx = fmaxf(mx, __uint_as_float(r[i]));
+      for (int u = 0; u < 4; ++u) mq[u] = fmaxf(__uint_as_float(r[2 * u]), __uint_as_float(r[2 * u + 1]));
+#pragma unroll
+      for (int i = 8; i < AT_N; i += 8)
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          mq[u] = max3(mq[u], __uint_as_float(r[i + 2 * u]), __uint_as_float(r[i + 2 * u + 1]));
+      const float mx = fmaxf(fmaxf(mq[0], mq[1]), fmaxf(mq[2], mq[3]));
       const float mx2 = mx * p.scale_log2;
       float alpha = 1.f;
       if (mx2 > m_use + 8.f) {
@@ -290,20 +319,22 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       }
       // P = exp2(s * scale - m) (masked keys give exp2(-inf) = 0), packed bf16 pairs
       // written over the S columns already read
-      float ls = 0.f;
+      float ls0 = 0.f, ls1 = 0.f;
 #pragma unroll
       for (int c = 0; c < AT_N / 32; ++c) {
         uint32_t pk[16];
 #pragma unroll
         for (int i = 0; i < 32; i += 2) {
-          const float a0 = ex2(fmaf(__uint_as_float(r[c * 32 + i]), p.scale_log2, -m_use));
-          const float a1 = ex2(fmaf(__uint_as_float(r[c * 32 + i + 1]), p.scale_log2, -m_use));
-          ls += a0 + a1;
+          float x0, x1;
+          fma2(x0, x1, __uint_as_float(r[c * 32 + i]), __uint_as_float(r[c * 32 + i + 1]),
+               p.scale_log2, -m_use);
+          const float a0 = ex2(x0), a1 = ex2(x1);
+          add2(ls0, ls1, a0, a1);
           pk[i / 2] = pack_bf16x2(a0, a1);
         }
         tmem_st16(s_addr + c * 16, pk);
       }
-      l += ls;
+      l += ls0 + ls1;
       // O_x holds PV of every earlier key tile (the S of this tile was issued after it);
       // rescale it before this tile's PV is issued
       if (j > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
