@@ -297,6 +297,13 @@ bag_status bag_rel_l1(bag_ctx* ctx, const void* a, const void* b, int dtype, lon
 bag_status bag_rel_l1_noalloc(const void* a, const void* b, int dtype, long rows, long cols,
                               float* out, void* cuda_stream);
 
+/* Failure-path check: launches one kernel whose mbarrier wait can never complete (no
+ * thread arrives on it), so its bounded wait gives up after the library's wait limit
+ * (about 2 s), records the sticky device error and returns; nothing faults or hangs.
+ * Returns BAG_EDEVICE_TIMEOUT once the stream reaches it; bag_run and bag_step report
+ * the sticky error until bag_reset.  For tests of the error path only. */
+bag_status bag_check_wait_timeout(bag_ctx* ctx);
+
 /* Skip path (plain residual reuse): out = h_in + R, fp32 device, n elements (n % 4 == 0). */
 bag_status bag_residual_add(bag_ctx* ctx, float* out, const float* h_in, const float* R, long n);
 

@@ -29,7 +29,8 @@ EXPORTS = ["bag_create", "bag_destroy", "bag_last_error", "bag_set_stream", "bag
            "bag_set_policy", "bag_set_budget", "bag_reset", "bag_step", "bag_run", "bag_run_host",
            "bag_get_weight", "bag_forward_block", "bag_prepare", "bag_launch_count",
            "bag_gemm_bf16", "bag_attention_bf16", "bag_ln_mod", "bag_residual_add",
-           "bag_profile_run", "bag_profile_launches", "bag_rel_l1", "bag_rel_l1_noalloc"]
+           "bag_profile_run", "bag_profile_launches", "bag_rel_l1", "bag_rel_l1_noalloc",
+           "bag_check_wait_timeout"]
 
 PROF_KINDS = ["gemm", "attention", "norm", "signal", "gate", "cache"]
 
@@ -96,6 +97,7 @@ def load(path=None):
         "bag_load_gate": ([_P, _P, _I, _P, _P], _I),
         "bag_set_policy": ([_P, _I, _P, ctypes.c_float], _I),
         "bag_set_budget": ([_P, _I], _I),
+        "bag_check_wait_timeout": ([_P], _I),
         "bag_reset": ([_P], _I),
         "bag_step": ([_P, _P, _I, ctypes.POINTER(Cond), _P, _P], _I),
         "bag_run": ([_P, _P, ctypes.POINTER(Cond), ctypes.POINTER(Stats)], _I),
@@ -211,6 +213,10 @@ class Context:
 
     def reset(self):
         self._chk(self.lib.bag_reset(self.h))
+
+    def check_wait_timeout(self):
+        """bag_check_wait_timeout: returns the status (BAG_EDEVICE_TIMEOUT expected)."""
+        return self.lib.bag_check_wait_timeout(self.h)
 
     def prepare(self, txt, pooled, txt_u=None, pooled_u=None):
         c = _cond(txt, pooled, txt_u, pooled_u)

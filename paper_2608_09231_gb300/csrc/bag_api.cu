@@ -1723,6 +1723,14 @@ bag_status bag_set_policy(bag_ctx* ctx, int policy, const uint8_t* host_mask, fl
   return BAG_OK;
 }
 
+bag_status bag_check_wait_timeout(bag_ctx* ctx) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  cudaError_t e = wait_timeout_probe(ctx->st, ctx->stream);
+  if (e != cudaSuccess) return leave(ctx, fail(ctx, BAG_ECUDA, std::string("probe: ") + cudaGetErrorString(e)));
+  return leave(ctx, check_device_error(ctx));
+}
+
 bag_status bag_set_budget(bag_ctx* ctx, int B) {
   if (!ctx) return BAG_EINVAL;
   if (B < 1 || B > ctx->T) return fail(ctx, BAG_EINVAL, "need 1 <= B <= T");

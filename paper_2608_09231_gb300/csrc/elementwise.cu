@@ -440,6 +440,24 @@ cudaError_t copy_rows_f32(const DevState* st, int flag_want, float* dst, long ld
 
 __global__ void advance_kernel(DevState* st) { st->t += 1; }
 
+// The bounded-wait failure path on purpose: the barrier expects one arrival that never
+// comes, mbar_wait gives up after kWaitLimitNs and the error is recorded like any
+// kernel's timed-out wait.
+__global__ void wait_timeout_kernel(DevState* st) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  abort_flag = 0;
+  mbar_init(&bar, 1);
+  fence_mbar_init();
+  if (!mbar_wait(&bar, 0, &abort_flag)) atomicOr(&st->err, 2);
+}
+
+cudaError_t wait_timeout_probe(DevState* st, cudaStream_t s) {
+  wait_timeout_kernel<<<1, 32, 0, s>>>(st);
+  return cudaGetLastError();
+}
+
 cudaError_t advance_step(DevState* st, cudaStream_t s) {
   advance_kernel<<<1, 1, 0, s>>>(st);
   return cudaGetLastError();

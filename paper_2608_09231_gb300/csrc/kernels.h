@@ -165,6 +165,8 @@ cudaError_t cache_reuse(const DevState* st, float* h_img, const float* h_in, con
 cudaError_t copy_rows_f32(const DevState* st, int flag_want, float* dst, long ldd, const void* src,
                           long lds, int src_bf16, int rows, int cols, cudaStream_t s);
 cudaError_t advance_step(DevState* st, cudaStream_t s);
+// one thread waits (bounded) on an mbarrier nothing arrives on, then sets st->err
+cudaError_t wait_timeout_probe(DevState* st, cudaStream_t s);
 cudaError_t sinusoid_all(void* out, int out_bf16, const double* sigma, int T, int dim, cudaStream_t s);
 cudaError_t expand_wan_mod(float* mod_all, const float* shared6d, const float* tables,
                            int T, int nblocks, int d, cudaStream_t s);

@@ -503,3 +503,28 @@ def test_unipc_budget_T_bit_exact_and_step_api(lib):
     torch.cuda.synchronize()
     assert torch.equal(xs, x)
     ctx.close()
+
+
+# ---------------------------------------------------------------------------
+# failure path: a bounded wait that runs out is reported, sticky, and cleared by reset
+# ---------------------------------------------------------------------------
+def test_bounded_wait_timeout_is_reported_and_sticky(lib):
+    import time
+    cfg = configs.get_config("tiny")
+    ctx = bag.create(cfg, T=4, B=2)
+    t0 = time.time()
+    st = ctx.check_wait_timeout()
+    dt = time.time() - t0
+    assert st == 5 and 1.0 < dt < 60.0, (st, dt)
+    assert "bounded wait" in lib.bag_last_error(ctx.h).decode()
+    inp = synth.make_inputs(cfg)
+    x, txt, pooled = _dev_inputs(cfg, inp)
+    with pytest.raises(bag.BagError) as ei:
+        ctx.run(x, txt, pooled)
+    assert ei.value.status == 5          # sticky until bag_reset
+    ctx.reset()
+    x, txt, pooled = _dev_inputs(cfg, inp)
+    m, _, nfe = ctx.run(x, txt, pooled)  # the context is usable again
+    torch.cuda.synchronize()
+    assert nfe == 2 and int(m.sum()) == 2
+    ctx.close()
