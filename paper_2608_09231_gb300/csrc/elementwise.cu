@@ -55,7 +55,11 @@ BAG_DEV void load4(const void* p, long off, int bf16, float* r) {
   }
 }
 
-__global__ void __launch_bounds__(LN_THREADS) ln_mod_kernel(const LnArgs a) {
+// VPT float4 per thread (cols <= 128 * 4 * VPT): the row stays in registers, and the
+// smallest VPT that holds it keeps the register count low enough for many rows per SM
+// (the kernel is latency-bound at low occupancy).
+template <int VPT>
+__global__ void __launch_bounds__(LN_THREADS, VPT <= 6 ? 8 : (VPT <= 10 ? 5 : 4)) ln_mod_kernel(const LnArgs a) {
   if (epi_skip(a.st, a.flag_want)) return;
   __shared__ float red[LN_THREADS / 32];
   const int row = blockIdx.x;
@@ -63,10 +67,10 @@ __global__ void __launch_bounds__(LN_THREADS) ln_mod_kernel(const LnArgs a) {
   const int t = a.st ? a.st->t : 0;
   const float* x = a.x + (long)row * a.ldx;
   const int nv = a.cols / 4;
-  float4 v[LN_MAXV];
+  float4 v[VPT];
   float s = 0.f;
 #pragma unroll
-  for (int i = 0; i < LN_MAXV; ++i) {
+  for (int i = 0; i < VPT; ++i) {
     const int c = threadIdx.x + i * LN_THREADS;
     if (c < nv) {
       v[i] = reinterpret_cast<const float4*>(x)[c];
@@ -76,7 +80,7 @@ __global__ void __launch_bounds__(LN_THREADS) ln_mod_kernel(const LnArgs a) {
   const float mean = block_sum(s, red) / (float)a.cols;
   float q = 0.f;
 #pragma unroll
-  for (int i = 0; i < LN_MAXV; ++i) {
+  for (int i = 0; i < VPT; ++i) {
     const int c = threadIdx.x + i * LN_THREADS;
     if (c < nv) {
       const float dx = v[i].x - mean, dy = v[i].y - mean, dz = v[i].z - mean, dw = v[i].w - mean;
@@ -91,7 +95,7 @@ __global__ void __launch_bounds__(LN_THREADS) ln_mod_kernel(const LnArgs a) {
   if (sc) sc += (long)t * a.mod_step;
   float sig_num = 0.f, sig_den = 0.f, sig_num2 = 0.f, sig_den2 = 0.f;
 #pragma unroll
-  for (int i = 0; i < LN_MAXV; ++i) {
+  for (int i = 0; i < VPT; ++i) {
     const int c = threadIdx.x + i * LN_THREADS;
     if (c < nv) {
       float y[4] = {(v[i].x - mean) * rstd, (v[i].y - mean) * rstd, (v[i].z - mean) * rstd,
@@ -154,7 +158,12 @@ __global__ void __launch_bounds__(LN_THREADS) ln_mod_kernel(const LnArgs a) {
 cudaError_t ln_mod(const LnArgs& a, cudaStream_t s) {
   if (a.rows <= 0) return cudaSuccess;
   if (a.cols % 4 != 0 || a.cols > LN_THREADS * 4 * LN_MAXV) return cudaErrorInvalidValue;
-  ln_mod_kernel<<<a.rows, LN_THREADS, 0, s>>>(a);
+  if (a.cols <= LN_THREADS * 4 * 6)
+    ln_mod_kernel<6><<<a.rows, LN_THREADS, 0, s>>>(a);
+  else if (a.cols <= LN_THREADS * 4 * 10)
+    ln_mod_kernel<10><<<a.rows, LN_THREADS, 0, s>>>(a);
+  else
+    ln_mod_kernel<LN_MAXV><<<a.rows, LN_THREADS, 0, s>>>(a);
   return cudaGetLastError();
 }
 
