@@ -24,6 +24,15 @@ BAG_DEV float gelu_tanh(float x) {
   return 0.5f * x * (1.0f + tanhf(u));
 }
 
+// The same with the hardware tanh approximation (tanh.approx.f32, relative error about
+// 2^-11), for outputs that are rounded to bf16 (relative step 2^-8) right after.
+BAG_DEV float gelu_tanh_fast(float x) {
+  const float k0 = 0.7978845608028654f, k1 = 0.044715f;
+  float t;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(k0 * (x + k1 * x * x * x)));
+  return 0.5f * x * (1.0f + t);
+}
+
 BAG_DEV float silu(float x) { return x / (1.0f + expf(-x)); }
 
 BAG_DEV uint32_t pack_bf16x2(float a, float b) {

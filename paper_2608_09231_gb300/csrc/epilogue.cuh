@@ -70,8 +70,13 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float r
       store_vals<NV>(e.out, (long)row * e.ldo + col0, v, e.out_bf16);
       break;
     case EPI_GELU:
+      if (e.out_bf16) {
 #pragma unroll
-      for (int j = 0; j < NV; ++j) v[j] = gelu_tanh(v[j]);
+        for (int j = 0; j < NV; ++j) v[j] = gelu_tanh_fast(v[j]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < NV; ++j) v[j] = gelu_tanh(v[j]);
+      }
       store_vals<NV>(e.out, (long)row * e.ldo + col0, v, e.out_bf16);
       break;
     case EPI_SILU:
@@ -84,7 +89,7 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float r
       const int region = lc / e.d;
       if (region >= 3) {
 #pragma unroll
-        for (int j = 0; j < NV; ++j) v[j] = gelu_tanh(v[j]);
+        for (int j = 0; j < NV; ++j) v[j] = e.act_bf16 ? gelu_tanh_fast(v[j]) : gelu_tanh(v[j]);
         store_vals<NV>(e.mlp, (long)row * e.ldm + (lc - 3 * e.d), v, e.act_bf16);
         break;
       }

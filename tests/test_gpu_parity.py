@@ -528,3 +528,29 @@ def test_bounded_wait_timeout_is_reported_and_sticky(lib):
     torch.cuda.synchronize()
     assert nfe == 2 and int(m.sum()) == 2
     ctx.close()
+
+
+# ---------------------------------------------------------------------------
+# the extensions together: guidance + QK-norm + UniPC + a six-input gate
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("name,over", [
+    ("flux_small", dict(guidance=3.0, qk_norm=True, sampler="unipc", shift=3.0, gate_kind="flux6")),
+    ("qwen_small", dict(guidance=4.0, qk_norm=True, gate_kind="wan6")),
+    ("wan_small", dict(guidance=5.0, gate_kind="wan6")),
+], ids=["flux_small-all", "qwen_small-cfg-qkn", "wan_small-cfg-unipc"])
+def test_extensions_combined_parity(name, over, lib):
+    cfg = configs.get_config(name, **over)
+    T, B = cfg["T"], cfg["budgets"][0]
+    inp = synth.make_inputs(cfg)
+    ctx, got, mask, log, nfe = _gpu_guided(cfg, T, B, inp)
+    ctx.close()
+    assert nfe == B and int(mask.sum()) == B and mask[0] == 1
+    W = synth.make_weights(cfg)
+    g = synth.make_gate_any(cfg["gate_seed"], cfg["gate_kind"])
+    steps = [None] + [float(v) for v in log[1:, 13]]
+    ref = O.sample(cfg, W, g, inp, T=T, B=B, drift_override=_gate_inputs(log),
+                   step_override=steps, guidance=cfg["guidance"])
+    assert list(mask) == ref["mask"]
+    rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
+    err = float(np.max(np.abs(got.astype(np.float64) - ref["x"])))
+    assert err <= TOL[cfg["dtype"]] * rms, (err, rms)
