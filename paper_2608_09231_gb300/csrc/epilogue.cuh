@@ -103,12 +103,27 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float r
       if (region < 2 && e.rope) {
         const int e0 = cc % e.dh;
         const float2* cs = e.rope + (long)jr * (e.dh / 2) + e0 / 2;
+        if constexpr (NV % 4 == 0) {
+          // two (cos, sin) pairs per 16-byte load (the table row offset is a multiple of
+          // NV / 2 pairs, so 16-byte aligned)
+          const float4* cs4 = reinterpret_cast<const float4*>(cs);
 #pragma unroll
-        for (int p = 0; p < NV / 2; ++p) {
-          const float2 r = __ldg(cs + p);
-          const float x0 = v[2 * p], x1 = v[2 * p + 1];
-          v[2 * p] = x0 * r.x - x1 * r.y;
-          v[2 * p + 1] = x0 * r.y + x1 * r.x;
+          for (int p = 0; p < NV / 4; ++p) {
+            const float4 r = __ldg(cs4 + p);
+            const float x0 = v[4 * p], x1 = v[4 * p + 1], x2 = v[4 * p + 2], x3 = v[4 * p + 3];
+            v[4 * p] = x0 * r.x - x1 * r.y;
+            v[4 * p + 1] = x0 * r.y + x1 * r.x;
+            v[4 * p + 2] = x2 * r.z - x3 * r.w;
+            v[4 * p + 3] = x2 * r.w + x3 * r.z;
+          }
+        } else {
+#pragma unroll
+          for (int p = 0; p < NV / 2; ++p) {
+            const float2 r = __ldg(cs + p);
+            const float x0 = v[2 * p], x1 = v[2 * p + 1];
+            v[2 * p] = x0 * r.x - x1 * r.y;
+            v[2 * p + 1] = x0 * r.y + x1 * r.x;
+          }
         }
       }
       if (region == 0) {

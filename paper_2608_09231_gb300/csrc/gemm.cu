@@ -152,10 +152,51 @@ static int tile_group_rows(int M, int BM, int K, int a_split) {
   return std::max(1, std::min(num_m, g));
 }
 
+// Per epilogue warp: a 32 x 33-word shared-memory tile for transposing V.
+constexpr int kVtScratchFloats = 32 * 33;
+constexpr int kVtScratchBytes = 4 * kVtScratchFloats * 4;  // four epilogue warps
+
+// V columns of a QKV projection with bf16 operands, stored transposed per head
+// (vt[(head * dh + e) * vpad + token]): the warp's 32 rows x 32 columns pass through
+// shared memory, so each lane writes one column's 32 consecutive tokens as four 16-byte
+// stores instead of 32 two-byte stores.  Rows past M (the last tile) and token offsets
+// that are not 16-byte aligned take per-element stores.
+BAG_DEV void store_vt_warp(const Epi& e, int row, int col, float* v, float* sbuf) {
+  const int lane = threadIdx.x & 31;
+  if (e.bias) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] += __ldg(e.bias + col + j);
+  }
+#pragma unroll
+  for (int j = 0; j < 32; ++j) sbuf[j * 33 + lane] = v[j];
+  __syncwarp();
+  float tc[32];
+#pragma unroll
+  for (int k = 0; k < 32; ++k) tc[k] = sbuf[lane * 33 + k];
+  __syncwarp();
+  const int row0 = row - lane;
+  const int jr0 = row0 + e.row_off;
+  const int cc = col + e.col_base - 2 * e.d + lane;  // this lane's column within V
+  __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(e.v) + (long)cc * e.vpad + jr0;
+  if (row0 + 31 < e.M && (jr0 & 7) == 0) {
+    uint4 w[4];
+    uint32_t* wp = reinterpret_cast<uint32_t*>(w);
+#pragma unroll
+    for (int k = 0; k < 16; ++k) wp[k] = pack_bf16x2(tc[2 * k], tc[2 * k + 1]);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) reinterpret_cast<uint4*>(dst)[k] = w[k];
+  } else {
+#pragma unroll
+    for (int k = 0; k < 32; ++k)
+      if (row0 + k < e.M) dst[k] = __float2bfloat16_rn(tc[k]);
+  }
+}
+
 // One thread's row of a BN-column accumulator in TMEM (lane base already in tb) through
-// the epilogue, columns col0 .. col0 + BN - 1.
+// the epilogue, columns col0 .. col0 + BN - 1.  vt_buf: this warp's transpose tile.
 template <int BN>
-BAG_DEV void drain_accumulator(const Epi& e, int t, int row, int col0, uint32_t tb) {
+BAG_DEV void drain_accumulator(const Epi& e, int t, int row, int col0, uint32_t tb, float* vt_buf) {
+  const bool vt_warp = e.kind == EPI_QKV && e.v_mode == 1 && e.act_bf16;
   if (e.qn_q) {
     // QK-norm: the tile holds whole heads (BN a multiple of dh, checked at launch); a
     // first pass over each q / k head takes its sum of squares (bias included), the
@@ -184,7 +225,10 @@ BAG_DEV void drain_accumulator(const Epi& e, int t, int row, int col0, uint32_t 
       for (int c = 0; c < dh; c += 32) {
         float v[32];
         tmem_ld32(tb + (uint32_t)(h0 + c), v);
-        epi_apply<32>(e, t, row, col + c, v, rs);
+        if (vt_warp && col + c < e.N && (col + c + e.col_base) / e.d == 2)
+          store_vt_warp(e, row, col + c, v, vt_buf);
+        else
+          epi_apply<32>(e, t, row, col + c, v, rs);
       }
     }
   } else {
@@ -192,7 +236,11 @@ BAG_DEV void drain_accumulator(const Epi& e, int t, int row, int col0, uint32_t 
     for (int c = 0; c < BN / 32; ++c) {
       float v[32];
       tmem_ld32(tb + (uint32_t)(c * 32), v);
-      epi_apply<32>(e, t, row, col0 + c * 32, v);
+      const int col = col0 + c * 32;
+      if (vt_warp && col < e.N && (col + e.col_base) / e.d == 2)
+        store_vt_warp(e, row, col, v, vt_buf);  // warp-uniform branch
+      else
+        epi_apply<32>(e, t, row, col, v);
     }
   }
 }
@@ -204,7 +252,7 @@ struct TcCfg {
   static constexpr int B_BYTES = BN * TC_BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int TMEM_COLS = 2 * BN;
-  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256 + kVtScratchBytes;
 };
 
 template <int BN>
@@ -229,6 +277,7 @@ __global__ void __launch_bounds__(192, 1)
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  float* vt_scratch = reinterpret_cast<float*>(smem + C::STAGES * C::STAGE_BYTES + 256);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -380,7 +429,7 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_after();
       const int row = mt * TC_BM + q * 32 + lane;
       const uint32_t tb = tmem_base + (uint32_t)(acc * BN) + ((uint32_t)(q * 32) << 16);
-      drain_accumulator<BN>(e, t, row, nt * BN, tb);
+      drain_accumulator<BN>(e, t, row, nt * BN, tb, vt_scratch + (warp - 2) * kVtScratchFloats);
       tc_fence_before();
       mbar_arrive(tempty + acc);
       acc ^= 1;
@@ -436,7 +485,7 @@ constexpr int PR_BM = 256, PR_BN = 256, PR_STAGES = 6;
 constexpr int PR_HALF_BYTES = 128 * TC_BK * 2;  // one CTA's A or W half-tile per k-block
 constexpr int PR_STAGE_BYTES = 2 * PR_HALF_BYTES;
 constexpr int PR_TMEM_COLS = 2 * PR_BN;         // double-buffered accumulator
-constexpr int PR_SMEM = PR_STAGES * PR_STAGE_BYTES + 1024 + 256;
+constexpr int PR_SMEM = PR_STAGES * PR_STAGE_BYTES + 1024 + 256 + kVtScratchBytes;
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
     gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
@@ -456,6 +505,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  float* vt_scratch = reinterpret_cast<float*>(smem + PR_STAGES * PR_STAGE_BYTES + 256);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -610,7 +660,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
       tc_fence_after();
       const int row = mt * PR_BM + (int)rank * 128 + q * 32 + lane;
       const uint32_t tb = tmem_base + (uint32_t)(acc * PR_BN) + ((uint32_t)(q * 32) << 16);
-      drain_accumulator<PR_BN>(e, t, row, nt * PR_BN, tb);
+      drain_accumulator<PR_BN>(e, t, row, nt * PR_BN, tb, vt_scratch + (warp - 2) * kVtScratchFloats);
       tc_fence_before();
       if (rank == 0)
         mbar_arrive(tempty + acc);
