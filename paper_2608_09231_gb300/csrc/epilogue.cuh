@@ -62,8 +62,20 @@ template <int NV>
 BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float rs = 1.f) {
   if (row >= e.M || col0 >= e.N) return;
   if (e.bias) {
+    if (NV % 4 == 0 && (reinterpret_cast<uintptr_t>(e.bias + col0) & 15) == 0) {
+      const float4* b4 = reinterpret_cast<const float4*>(e.bias + col0);
 #pragma unroll
-    for (int j = 0; j < NV; ++j) v[j] += __ldg(e.bias + col0 + j);
+      for (int j = 0; j < NV; j += 4) {
+        const float4 b = __ldg(b4 + j / 4);
+        v[j] += b.x;
+        v[j + 1] += b.y;
+        v[j + 2] += b.z;
+        v[j + 3] += b.w;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < NV; ++j) v[j] += __ldg(e.bias + col0 + j);
+    }
   }
   switch (e.kind) {
     case EPI_STORE:
@@ -149,14 +161,15 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float r
     case EPI_GATED_RES: {
       const float* g = e.gate + (long)t * e.gate_step + col0;
       float* r = e.resid + (long)row * e.ldr + col0;
-      if constexpr (NV % 4 == 0) {
+      if (NV % 4 == 0 && ((reinterpret_cast<uintptr_t>(g) | reinterpret_cast<uintptr_t>(r)) & 15) == 0) {
 #pragma unroll
         for (int j = 0; j < NV; j += 4) {
+          const float4 g4 = __ldg(reinterpret_cast<const float4*>(g + j));
           float4 h = *reinterpret_cast<float4*>(r + j);
-          h.x += __ldg(g + j) * v[j];
-          h.y += __ldg(g + j + 1) * v[j + 1];
-          h.z += __ldg(g + j + 2) * v[j + 2];
-          h.w += __ldg(g + j + 3) * v[j + 3];
+          h.x += g4.x * v[j];
+          h.y += g4.y * v[j + 1];
+          h.z += g4.z * v[j + 2];
+          h.w += g4.w * v[j + 3];
           *reinterpret_cast<float4*>(r + j) = h;
         }
       } else {
