@@ -56,11 +56,9 @@ BAG_DEV void store_vals(void* base, long idx, const float* v, int bf16) {
 // Apply the epilogue to NV consecutive accumulators v[0..NV) of output row `row`,
 // columns [col0, col0 + NV).  NV is even and col0 is a multiple of NV; the chunk never
 // straddles a q/k/v/mlp boundary (those are multiples of 64 columns).
-// rs: EPI_QKV with QK-norm, 1 / RMS of the head that columns col0 .. col0 + NV - 1 of
-// this row belong to (computed by the caller over the whole head).
+// Bias of the output columns col0 .. col0 + NV - 1 (16-byte loads when aligned).
 template <int NV>
-BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float rs = 1.f) {
-  if (row >= e.M || col0 >= e.N) return;
+BAG_DEV void epi_add_bias(const Epi& e, int col0, float* v) {
   if (e.bias) {
     if (NV % 4 == 0 && (reinterpret_cast<uintptr_t>(e.bias + col0) & 15) == 0) {
       const float4* b4 = reinterpret_cast<const float4*>(e.bias + col0);
@@ -77,6 +75,51 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float r
       for (int j = 0; j < NV; ++j) v[j] += __ldg(e.bias + col0 + j);
     }
   }
+}
+
+// EPI_QKV q / k columns (region 0 / 1): per-head RMSNorm (when the block has it), then
+// the rotation of joint-sequence row jr; cc is the column within the region.
+template <int NV>
+BAG_DEV void epi_qk_transform(const Epi& e, int jr, int cc, int region, float* v, float rs) {
+  if (region < 2 && e.qn_q) {  // per-head RMSNorm of q and k, before the rotation
+    const float* w = (region == 0 ? e.qn_q : e.qn_k) + cc % e.dh;
+#pragma unroll
+    for (int j = 0; j < NV; ++j) v[j] = v[j] * rs * __ldg(w + j);
+  }
+  if (region < 2 && e.rope) {
+    const int e0 = cc % e.dh;
+    const float2* cs = e.rope + (long)jr * (e.dh / 2) + e0 / 2;
+    if constexpr (NV % 4 == 0) {
+      // two (cos, sin) pairs per 16-byte load (the table row offset is a multiple of
+      // NV / 2 pairs, so 16-byte aligned)
+      const float4* cs4 = reinterpret_cast<const float4*>(cs);
+#pragma unroll
+      for (int p = 0; p < NV / 4; ++p) {
+        const float4 r = __ldg(cs4 + p);
+        const float x0 = v[4 * p], x1 = v[4 * p + 1], x2 = v[4 * p + 2], x3 = v[4 * p + 3];
+        v[4 * p] = x0 * r.x - x1 * r.y;
+        v[4 * p + 1] = x0 * r.y + x1 * r.x;
+        v[4 * p + 2] = x2 * r.z - x3 * r.w;
+        v[4 * p + 3] = x2 * r.w + x3 * r.z;
+      }
+    } else {
+#pragma unroll
+      for (int p = 0; p < NV / 2; ++p) {
+        const float2 r = __ldg(cs + p);
+        const float x0 = v[2 * p], x1 = v[2 * p + 1];
+        v[2 * p] = x0 * r.x - x1 * r.y;
+        v[2 * p + 1] = x0 * r.y + x1 * r.x;
+      }
+    }
+  }
+}
+
+// rs: EPI_QKV with QK-norm, 1 / RMS of the head that columns col0 .. col0 + NV - 1 of
+// this row belong to (computed by the caller over the whole head).
+template <int NV>
+BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float rs = 1.f) {
+  if (row >= e.M || col0 >= e.N) return;
+  epi_add_bias<NV>(e, col0, v);
   switch (e.kind) {
     case EPI_STORE:
       store_vals<NV>(e.out, (long)row * e.ldo + col0, v, e.out_bf16);
@@ -107,37 +150,7 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float r
       }
       const int jr = row + e.row_off;  // joint-sequence row
       const int cc = lc - region * e.d;
-      if (region < 2 && e.qn_q) {  // per-head RMSNorm of q and k, before the rotation
-        const float* w = (region == 0 ? e.qn_q : e.qn_k) + cc % e.dh;
-#pragma unroll
-        for (int j = 0; j < NV; ++j) v[j] = v[j] * rs * __ldg(w + j);
-      }
-      if (region < 2 && e.rope) {
-        const int e0 = cc % e.dh;
-        const float2* cs = e.rope + (long)jr * (e.dh / 2) + e0 / 2;
-        if constexpr (NV % 4 == 0) {
-          // two (cos, sin) pairs per 16-byte load (the table row offset is a multiple of
-          // NV / 2 pairs, so 16-byte aligned)
-          const float4* cs4 = reinterpret_cast<const float4*>(cs);
-#pragma unroll
-          for (int p = 0; p < NV / 4; ++p) {
-            const float4 r = __ldg(cs4 + p);
-            const float x0 = v[4 * p], x1 = v[4 * p + 1], x2 = v[4 * p + 2], x3 = v[4 * p + 3];
-            v[4 * p] = x0 * r.x - x1 * r.y;
-            v[4 * p + 1] = x0 * r.y + x1 * r.x;
-            v[4 * p + 2] = x2 * r.z - x3 * r.w;
-            v[4 * p + 3] = x2 * r.w + x3 * r.z;
-          }
-        } else {
-#pragma unroll
-          for (int p = 0; p < NV / 2; ++p) {
-            const float2 r = __ldg(cs + p);
-            const float x0 = v[2 * p], x1 = v[2 * p + 1];
-            v[2 * p] = x0 * r.x - x1 * r.y;
-            v[2 * p + 1] = x0 * r.y + x1 * r.x;
-          }
-        }
-      }
+      if (region < 2) epi_qk_transform<NV>(e, jr, cc, region, v, rs);
       if (region == 0) {
         store_vals<NV>(e.q, (long)jr * e.ldqk + cc, v, e.act_bf16);
       } else if (region == 1) {
