@@ -37,6 +37,30 @@ BAG_DEV float block_sum(float v, float* red) {
   return s;
 }
 
+// Four block-wide sums at once (one pair of barriers instead of four).
+BAG_DEV float4 block_sum4(float4 v, float4* red) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    v.x += __shfl_xor_sync(0xffffffffu, v.x, off);
+    v.y += __shfl_xor_sync(0xffffffffu, v.y, off);
+    v.z += __shfl_xor_sync(0xffffffffu, v.z, off);
+    v.w += __shfl_xor_sync(0xffffffffu, v.w, off);
+  }
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+  for (int w = 0; w < LN_THREADS / 32; ++w) {
+    s.x += red[w].x;
+    s.y += red[w].y;
+    s.z += red[w].z;
+    s.w += red[w].w;
+  }
+  return s;
+}
+
 BAG_DEV void load4(const void* p, long off, int bf16, float* r) {
   if (bf16) {
     const uint2 u = *reinterpret_cast<const uint2*>(reinterpret_cast<const __nv_bfloat16*>(p) + off);
@@ -142,16 +166,9 @@ __global__ void __launch_bounds__(LN_THREADS, VPT <= 6 ? 8 : (VPT <= 10 ? 5 : 4)
     }
   }
   if (a.sig_on) {
-    const float n = block_sum(sig_num, red);
-    const float d = block_sum(sig_den, red);
-    const float n2 = block_sum(sig_num2, red);
-    const float d2 = block_sum(sig_den2, red);
-    if (threadIdx.x == 0) {
-      a.sig_partial[4 * row] = n;
-      a.sig_partial[4 * row + 1] = d;
-      a.sig_partial[4 * row + 2] = n2;
-      a.sig_partial[4 * row + 3] = d2;
-    }
+    __shared__ float4 red4[LN_THREADS / 32];
+    const float4 t4 = block_sum4(make_float4(sig_num, sig_den, sig_num2, sig_den2), red4);
+    if (threadIdx.x == 0) reinterpret_cast<float4*>(a.sig_partial)[row] = t4;
   }
 }
 
