@@ -170,10 +170,10 @@ def _bf16_tensor(seed, shape, std=1.0):
 
 
 # (4096, 3072, 3072), (1000, 19456, 192) and (4100, 4864, 320) have enough 256 x 256
-# tiles for the CTA-pair kernel (the last two with a ragged final row tile)
+# tiles for the CTA-pair kernel (the last three with a ragged final row tile)
 @pytest.mark.parametrize("M,N,K", [(300, 256, 128), (129, 64, 64), (1000, 384, 512),
                                    (77, 512, 256), (4096, 3072, 3072), (50, 1024, 320),
-                                   (1000, 19456, 192), (4100, 4864, 320)])
+                                   (1000, 19456, 192), (4100, 4864, 320), (7000, 3072, 256)])
 @pytest.mark.parametrize("simt", [0, 1])
 def test_gemm_bf16_against_fp64(M, N, K, simt, lib):
     ctx = bag.create("tiny", T=2, B=1)
@@ -192,7 +192,7 @@ def test_gemm_bf16_against_fp64(M, N, K, simt, lib):
     ctx.close()
 
 
-@pytest.mark.parametrize("M,N,K", [(257, 128, 192), (700, 19456, 128)])
+@pytest.mark.parametrize("M,N,K", [(257, 128, 192), (700, 19456, 128), (7000, 3072, 128)])
 def test_gemm_gelu_epilogue(M, N, K, lib):
     ctx = bag.create("tiny", T=2, B=1)
     a, A = _bf16_tensor(4, (M, K))
@@ -554,3 +554,24 @@ def test_extensions_combined_parity(name, over, lib):
     rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
     err = float(np.max(np.abs(got.astype(np.float64) - ref["x"])))
     assert err <= TOL[cfg["dtype"]] * rms, (err, rms)
+
+
+def test_set_budget_between_samples(lib):
+    """bag_set_budget: the next sample spends exactly the new budget under Algorithm 2,
+    and a static evenly spaced schedule is recomputed for it."""
+    cfg = configs.get_config("tiny_ragged")
+    T = cfg["T"]
+    ctx = bag.create(cfg, T=T, B=2)
+    for B in (2, 5, 1, T):
+        ctx.set_budget(B)
+        _, _, m, _, nfe = _gpu_sample(cfg, T, B, ctx=ctx)
+        assert nfe == B and int(m.sum()) == B and m[0] == 1
+    ctx.set_policy(bag.POLICY_STATIC_UNIFORM)
+    for B in (3, 4):
+        ctx.set_budget(B)
+        _, _, m, _, nfe = _gpu_sample(cfg, T, B, ctx=ctx)
+        assert list(m) == O.static_uniform_schedule(B, T) and nfe == B
+    with pytest.raises(bag.BagError) as ei:
+        ctx.set_budget(T + 1)
+    assert ei.value.status == 1
+    ctx.close()
