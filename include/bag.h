@@ -133,7 +133,10 @@ typedef struct bag_ctx bag_ctx;
  * Sec. 3.1: ||m||_1 = B with m_0 = 1).  Allocates and seeds all weights on the current
  * CUDA device from arch->weight_seed (SplitMix64 counter generator), seeds the gate
  * from arch->gate_seed, and allocates every activation buffer the step needs, so that
- * no later call allocates.  *out receives the context (NULL on failure).
+ * no later call allocates.  *out receives the context (NULL on failure).  Consecutive
+ * kernels of a step are launched with programmatic stream serialization (each kernel
+ * waits on the device for its predecessor); the environment variable BAG_PDL=0, read
+ * here, launches them with plain stream order instead.
  * Errors: EINVAL (bad arch/T/B), ENOMEM, ECUDA, EUNSUPPORTED. */
 bag_status bag_create(const bag_arch* arch, int T, int B, bag_ctx** out);
 

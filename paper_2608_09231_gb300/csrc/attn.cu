@@ -22,6 +22,7 @@ BAG_DEV float ldv(const void* p, long i) {
 // are staged in shared memory (K transposed so that lane j reads key j's column).
 template <typename T, int DH>
 __global__ void __launch_bounds__(128) attn_simt_kernel(const AttnArgs a) {
+  grid_dep_sync();
   if (epi_skip(a.st, a.flag_want)) return;
   constexpr int QPW = 4, QPB = 16, KT = 32, R = DH / 32;
   __shared__ float Qs[QPB][DH];
@@ -110,14 +111,14 @@ cudaError_t attention(const AttnArgs& a, int* err, cudaStream_t s, int force_sim
   dim3 grid((a.nq + 15) / 16, a.heads);
   if (a.dh == 64) {
     if (a.bf16)
-      attn_simt_kernel<__nv_bfloat16, 64><<<grid, 128, 0, s>>>(a);
+      launch_kernel(attn_simt_kernel<__nv_bfloat16, 64>, grid, 128, 0, s, a);
     else
-      attn_simt_kernel<float, 64><<<grid, 128, 0, s>>>(a);
+      launch_kernel(attn_simt_kernel<float, 64>, grid, 128, 0, s, a);
   } else if (a.dh == 128) {
     if (a.bf16)
-      attn_simt_kernel<__nv_bfloat16, 128><<<grid, 128, 0, s>>>(a);
+      launch_kernel(attn_simt_kernel<__nv_bfloat16, 128>, grid, 128, 0, s, a);
     else
-      attn_simt_kernel<float, 128><<<grid, 128, 0, s>>>(a);
+      launch_kernel(attn_simt_kernel<float, 128>, grid, 128, 0, s, a);
   } else {
     return cudaErrorInvalidValue;
   }

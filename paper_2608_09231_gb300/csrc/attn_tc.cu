@@ -120,6 +120,7 @@ BAG_DEV void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint3
 __global__ void __launch_bounds__(AT_THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, const AttnTcParams p) {
+  grid_dep_sync();
   if (epi_skip(p.st, p.flag_want)) return;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -407,7 +408,7 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t s) {
   p.flag_want = a.flag_want;
   p.err = err;
   dim3 grid((a.nq + 2 * AT_M - 1) / (2 * AT_M), a.heads);
-  attn_tc_kernel<<<grid, AT_THREADS, AT_SMEM, s>>>(tq, tk, tv, p);
+  launch_kernel(attn_tc_kernel, grid, AT_THREADS, AT_SMEM, s, tq, tk, tv, p);
   return cudaGetLastError();
 }
 

@@ -13,6 +13,7 @@
 //   suffix : final LN-mod + projection fused with the Euler update, t += 1
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 #include <cstdio>
 #include <cstring>
 #include <map>
@@ -157,6 +158,7 @@ struct bag_ctx {
   cudaGraphExec_t exec = nullptr;
   cudaStream_t cap_stream = nullptr;
   int use_graph = 1;
+  bool pdl = true;  // programmatic dependent launch between the kernels of a segment
   long n_prefix = 0, n_full = 0, n_skip = 0, n_suffix = 0, n_prepare = 0;
   long launches = 0;
 
@@ -178,6 +180,7 @@ struct bag_ctx {
 };
 
 static std::string g_create_error;
+thread_local bool bag::g_pdl = false;
 
 void bag::set_global_error(const std::string& msg) { g_create_error = msg; }
 
@@ -694,11 +697,19 @@ static int prof_event(bag_ctx* ctx) {
   return (int)ctx->ev_used++;
 }
 
+// One enqueued segment of kernels on one stream (a step's prefix, a body of the
+// conditional, the suffix, a block, the per-sample preparation).  Every launch after
+// the segment's first is made with programmatic stream serialization unless profiling
+// (whose events sit between the kernels) or the context turned it off.
 struct Enq {
   bag_ctx* ctx;
   cudaStream_t s;
   long* count;
   cudaError_t e = cudaSuccess;
+  Enq(bag_ctx* c, cudaStream_t st, long* n) : ctx(c), s(st), count(n) { g_pdl = false; }
+  ~Enq() { g_pdl = false; }
+  Enq(const Enq&) = delete;
+  Enq& operator=(const Enq&) = delete;
   int pk = -1, pe0 = -1, pm = 0, pn = 0, pkk = 0, pv = 0;
   double pf = 0, pb = 0;
   // announce the next launch (kind, algorithmic flops and bytes, shape, kernel variant)
@@ -719,6 +730,7 @@ struct Enq {
   void chk(cudaError_t r) {
     if (e == cudaSuccess && r != cudaSuccess) e = r;
     if (count) ++*count;
+    g_pdl = ctx->pdl && !ctx->profiling;
     if (pk >= 0) {
       const int pe1 = prof_event(ctx);
       if (pe1 >= 0) {
@@ -1627,6 +1639,7 @@ bag_status bag_create(const bag_arch* arch, int T, int B, bag_ctx** out) {
   ctx->act_bf16 = arch->dtype == BAG_BF16;
   ctx->act_size = ctx->act_bf16 ? 2 : 4;
   ctx->thr = (float)std::log((double)arch->tau / (1.0 - (double)arch->tau));
+  if (const char* v = std::getenv("BAG_PDL")) ctx->pdl = std::atoi(v) != 0;
   if (arch->kind == BAG_KIND_WAN) {
     ctx->nblk = arch->n_wan;
     ctx->blocks.assign(ctx->nblk, Block{});

@@ -14,6 +14,17 @@
 
 namespace bag {
 
+// Programmatic dependent launch.  A kernel launched with programmatic stream
+// serialization may be scheduled while the previous kernel on its stream is still
+// running; griddepcontrol.wait blocks until that kernel has completed and its memory
+// writes are visible, and launch_dependents lets the next kernel's CTAs be scheduled
+// early (they wait the same way).  Every kernel calls this before its first access to
+// global memory; in a kernel launched without the attribute both are no-ops.
+__device__ __forceinline__ void grid_dep_sync() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---------------------------------------------------------------------------
 // numeric helpers
 // ---------------------------------------------------------------------------

@@ -84,6 +84,7 @@ BAG_DEV void load4(const void* p, long off, int bf16, float* r) {
 // (the kernel is latency-bound at low occupancy).
 template <int VPT>
 __global__ void __launch_bounds__(LN_THREADS, VPT <= 6 ? 8 : (VPT <= 10 ? 5 : 4)) ln_mod_kernel(const LnArgs a) {
+  grid_dep_sync();
   if (epi_skip(a.st, a.flag_want)) return;
   __shared__ float red[LN_THREADS / 32];
   const int row = blockIdx.x;
@@ -176,17 +177,18 @@ cudaError_t ln_mod(const LnArgs& a, cudaStream_t s) {
   if (a.rows <= 0) return cudaSuccess;
   if (a.cols % 4 != 0 || a.cols > LN_THREADS * 4 * LN_MAXV) return cudaErrorInvalidValue;
   if (a.cols <= LN_THREADS * 4 * 6)
-    ln_mod_kernel<6><<<a.rows, LN_THREADS, 0, s>>>(a);
+    launch_kernel(ln_mod_kernel<6>, a.rows, LN_THREADS, 0, s, a);
   else if (a.cols <= LN_THREADS * 4 * 10)
-    ln_mod_kernel<10><<<a.rows, LN_THREADS, 0, s>>>(a);
+    launch_kernel(ln_mod_kernel<10>, a.rows, LN_THREADS, 0, s, a);
   else
-    ln_mod_kernel<LN_MAXV><<<a.rows, LN_THREADS, 0, s>>>(a);
+    launch_kernel(ln_mod_kernel<LN_MAXV>, a.rows, LN_THREADS, 0, s, a);
   return cudaGetLastError();
 }
 
 // Standalone relative-L1 partial sums (same reduction as the fused signal).
 __global__ void __launch_bounds__(LN_THREADS) rel_l1_kernel(const void* a, const void* b, int bf16,
                                                             long cols, float* partial) {
+  grid_dep_sync();
   __shared__ float red[LN_THREADS / 32];
   const long row = blockIdx.x;
   float n = 0.f, d = 0.f;
@@ -214,13 +216,14 @@ __global__ void __launch_bounds__(LN_THREADS) rel_l1_kernel(const void* a, const
 cudaError_t rel_l1_partials(const void* a, const void* b, int a_bf16, long rows, long cols,
                             float* partial, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
-  rel_l1_kernel<<<(unsigned)rows, LN_THREADS, 0, s>>>(a, b, a_bf16, cols, partial);
+  launch_kernel(rel_l1_kernel, (unsigned)rows, LN_THREADS, 0, s, a, b, a_bf16, cols, partial);
   return cudaGetLastError();
 }
 
 // out[0] = sum(num) / sum(den), out[1] = sum(num), out[2] = sum(den) over the per-row
 // partials, summed in the same fixed order as the gate kernel's drift reduction.
 __global__ void rel_l1_finalize_kernel(const float* partial, long rows, float* out) {
+  grid_dep_sync();
   const int lane = threadIdx.x;
   float num = 0.f, den = 0.f;
   for (long r = lane; r < rows; r += 32) {
@@ -240,7 +243,7 @@ __global__ void rel_l1_finalize_kernel(const float* partial, long rows, float* o
 }
 
 cudaError_t rel_l1_finalize(const float* partial, long rows, float* out, cudaStream_t s) {
-  rel_l1_finalize_kernel<<<1, 32, 0, s>>>(partial, rows, out);
+  launch_kernel(rel_l1_finalize_kernel, 1, 32, 0, s, partial, rows, out);
   return cudaGetLastError();
 }
 
@@ -271,6 +274,7 @@ __global__ void gate_kernel(DevState* st, const float* partial, int rows, const 
                             int kind, float thr, int T, int B, int policy, const uint8_t* pmask,
                             float delta, float* log, cudaGraphConditionalHandle handle,
                             int use_cond) {
+  grid_dep_sync();
   const int lane = threadIdx.x;
   const int t = st->t, c = st->c, t_last = st->t_last;
   float num = 0.f, den = 0.f, num2 = 0.f, den2 = 0.f;
@@ -370,9 +374,8 @@ cudaError_t gate_step(DevState* st, const float* sig_partial, int sig_rows, cons
                       int gate_kind, float thr, int T, int B, int policy, const uint8_t* policy_mask,
                       float delta, float* log, unsigned long long cond_handle, int use_cond,
                       cudaStream_t s) {
-  gate_kernel<<<1, 32, 0, s>>>(st, sig_partial, sig_rows, gate_params, gate_kind, thr, T, B, policy,
-                               policy_mask, delta, log, (cudaGraphConditionalHandle)cond_handle,
-                               use_cond);
+  launch_kernel(gate_kernel, 1, 32, 0, s, st, sig_partial, sig_rows, gate_params, gate_kind, thr, T, B,
+                policy, policy_mask, delta, log, (cudaGraphConditionalHandle)cond_handle, use_cond);
   return cudaGetLastError();
 }
 
@@ -382,6 +385,7 @@ cudaError_t gate_step(DevState* st, const float* sig_partial, int sig_rows, cons
 __global__ void cache_refresh_kernel(const DevState* st, int flag_want, const float4* h_img,
                                      const float4* h_in, float4* R, long n4, uint4* m_last,
                                      const uint4* m_cur, long m16) {
+  grid_dep_sync();
   if (epi_skip(st, flag_want)) return;
   const long stride = (long)gridDim.x * blockDim.x;
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
@@ -393,6 +397,7 @@ __global__ void cache_refresh_kernel(const DevState* st, int flag_want, const fl
 
 __global__ void cache_reuse_kernel(const DevState* st, int flag_want, float4* h_img,
                                    const float4* h_in, const float4* R, long n4) {
+  grid_dep_sync();
   if (epi_skip(st, flag_want)) return;
   const long stride = (long)gridDim.x * blockDim.x;
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += stride) {
@@ -422,19 +427,19 @@ cudaError_t cache_refresh(const DevState* st, const float* h_img, const float* h
   if (n % 4 != 0) return cudaErrorInvalidValue;
   const long mbytes = m_n * (m_bf16 ? 2 : 4);
   if (mbytes % 16 != 0) return cudaErrorInvalidValue;
-  cache_refresh_kernel<<<grid_for(n / 4, 256), 256, 0, s>>>(
-      st, flag_want, reinterpret_cast<const float4*>(h_img), reinterpret_cast<const float4*>(h_in),
-      reinterpret_cast<float4*>(R), n / 4, reinterpret_cast<uint4*>(m_last),
-      reinterpret_cast<const uint4*>(m_cur), mbytes / 16);
+  launch_kernel(cache_refresh_kernel, grid_for(n / 4, 256), 256, 0, s, st, flag_want,
+                reinterpret_cast<const float4*>(h_img), reinterpret_cast<const float4*>(h_in),
+                reinterpret_cast<float4*>(R), n / 4, reinterpret_cast<uint4*>(m_last),
+                reinterpret_cast<const uint4*>(m_cur), mbytes / 16);
   return cudaGetLastError();
 }
 
 cudaError_t cache_reuse(const DevState* st, float* h_img, const float* h_in, const float* R,
                         long n, int flag_want, cudaStream_t s) {
   if (n % 4 != 0) return cudaErrorInvalidValue;
-  cache_reuse_kernel<<<grid_for(n / 4, 256), 256, 0, s>>>(
-      st, flag_want, reinterpret_cast<float4*>(h_img), reinterpret_cast<const float4*>(h_in),
-      reinterpret_cast<const float4*>(R), n / 4);
+  launch_kernel(cache_reuse_kernel, grid_for(n / 4, 256), 256, 0, s, st, flag_want,
+                reinterpret_cast<float4*>(h_img), reinterpret_cast<const float4*>(h_in),
+                reinterpret_cast<const float4*>(R), n / 4);
   return cudaGetLastError();
 }
 
@@ -447,6 +452,7 @@ cudaError_t residual_add(float* out, const float* a, const float* b, long n, cud
 // ---------------------------------------------------------------------------
 __global__ void copy_rows_kernel(const DevState* st, int flag_want, float* dst, long ldd,
                                  const void* src, long lds, int src_bf16, int rows, int cols) {
+  grid_dep_sync();
   if (epi_skip(st, flag_want)) return;
   const long n = (long)rows * cols;
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
@@ -459,17 +465,21 @@ __global__ void copy_rows_kernel(const DevState* st, int flag_want, float* dst, 
 cudaError_t copy_rows_f32(const DevState* st, int flag_want, float* dst, long ldd, const void* src,
                           long lds, int src_bf16, int rows, int cols, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
-  copy_rows_kernel<<<grid_for((long)rows * cols, 256), 256, 0, s>>>(st, flag_want, dst, ldd, src,
-                                                                    lds, src_bf16, rows, cols);
+  launch_kernel(copy_rows_kernel, grid_for((long)rows * cols, 256), 256, 0, s, st, flag_want, dst, ldd,
+                src, lds, src_bf16, rows, cols);
   return cudaGetLastError();
 }
 
-__global__ void advance_kernel(DevState* st) { st->t += 1; }
+__global__ void advance_kernel(DevState* st) {
+  grid_dep_sync();
+  st->t += 1;
+}
 
 // The bounded-wait failure path on purpose: the barrier expects one arrival that never
 // comes, mbar_wait gives up after kWaitLimitNs and the error is recorded like any
 // kernel's timed-out wait.
 __global__ void wait_timeout_kernel(DevState* st) {
+  grid_dep_sync();
   __shared__ uint64_t bar;
   __shared__ int abort_flag;
   if (threadIdx.x != 0) return;
@@ -480,18 +490,19 @@ __global__ void wait_timeout_kernel(DevState* st) {
 }
 
 cudaError_t wait_timeout_probe(DevState* st, cudaStream_t s) {
-  wait_timeout_kernel<<<1, 32, 0, s>>>(st);
+  launch_kernel(wait_timeout_kernel, 1, 32, 0, s, st);
   return cudaGetLastError();
 }
 
 cudaError_t advance_step(DevState* st, cudaStream_t s) {
-  advance_kernel<<<1, 1, 0, s>>>(st);
+  launch_kernel(advance_kernel, 1, 1, 0, s, st);
   return cudaGetLastError();
 }
 
 // Sinusoidal features of 1000 * sigma_t, sigma_t = 1 - t/T, for every step t < T:
 // [cos(1000 sigma_t f_j), sin(1000 sigma_t f_j)], f_j = exp(-ln(10000) j / (dim/2)).
 __global__ void sinusoid_kernel(void* out, int out_bf16, const double* sigma, int T, int dim) {
+  grid_dep_sync();
   const int t = blockIdx.x, j = threadIdx.x;
   const int half = dim / 2;
   if (t >= T || j >= dim) return;
@@ -507,7 +518,7 @@ __global__ void sinusoid_kernel(void* out, int out_bf16, const double* sigma, in
 }
 
 cudaError_t sinusoid_all(void* out, int out_bf16, const double* sigma, int T, int dim, cudaStream_t s) {
-  sinusoid_kernel<<<T, dim, 0, s>>>(out, out_bf16, sigma, T, dim);
+  launch_kernel(sinusoid_kernel, T, dim, 0, s, out, out_bf16, sigma, T, dim);
   return cudaGetLastError();
 }
 
@@ -516,6 +527,7 @@ cudaError_t sinusoid_all(void* out, int out_bf16, const double* sigma, int T, in
 // mod_all:  [T][nblocks*6d + 2d].
 __global__ void expand_wan_kernel(float* mod_all, const float* shared8d, const float* tables,
                                   int T, int nblocks, int d) {
+  grid_dep_sync();
   const long per = (long)nblocks * 6 * d + 2 * d;
   const long n = (long)T * per;
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
@@ -532,12 +544,13 @@ __global__ void expand_wan_kernel(float* mod_all, const float* shared8d, const f
 
 cudaError_t expand_wan_mod(float* mod_all, const float* shared8d, const float* tables, int T,
                            int nblocks, int d, cudaStream_t s) {
-  expand_wan_kernel<<<grid_for((long)T * nblocks * 6 * d, 256), 256, 0, s>>>(mod_all, shared8d,
-                                                                           tables, T, nblocks, d);
+  launch_kernel(expand_wan_kernel, grid_for((long)T * nblocks * 6 * d, 256), 256, 0, s, mod_all,
+                shared8d, tables, T, nblocks, d);
   return cudaGetLastError();
 }
 
 __global__ void split_bf16_kernel(__nv_bfloat16* dst, const float* src, long rows, long cols) {
+  grid_dep_sync();
   const long n = rows * cols;
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
     const long r = i / cols, c = i % cols;
@@ -550,18 +563,19 @@ __global__ void split_bf16_kernel(__nv_bfloat16* dst, const float* src, long row
 
 cudaError_t split_bf16(__nv_bfloat16* dst, const float* src, long rows, long cols, cudaStream_t s) {
   if (rows * cols <= 0) return cudaSuccess;
-  split_bf16_kernel<<<grid_for(rows * cols, 256), 256, 0, s>>>(dst, src, rows, cols);
+  launch_kernel(split_bf16_kernel, grid_for(rows * cols, 256), 256, 0, s, dst, src, rows, cols);
   return cudaGetLastError();
 }
 
 __global__ void to_bf16_kernel(__nv_bfloat16* dst, const float* src, long n) {
+  grid_dep_sync();
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x)
     dst[i] = __float2bfloat16_rn(src[i]);
 }
 
 cudaError_t to_bf16(__nv_bfloat16* dst, const float* src, long n, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
-  to_bf16_kernel<<<grid_for(n, 256), 256, 0, s>>>(dst, src, n);
+  launch_kernel(to_bf16_kernel, grid_for(n, 256), 256, 0, s, dst, src, n);
   return cudaGetLastError();
 }
 
@@ -575,6 +589,7 @@ BAG_DEV uint64_t sm64_mix(uint64_t z) {
 }
 
 __global__ void fill_synth_kernel(void* dst, long n, uint64_t start, float offset, float c32, int bf16) {
+  grid_dep_sync();
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x) {
     const uint64_t u = sm64_mix(start + (uint64_t)(i + 1) * 0x9E3779B97F4A7C15ull);
     const long q = (long)(u & 0xFFFF) + (long)((u >> 16) & 0xFFFF) + (long)((u >> 32) & 0xFFFF) +
@@ -591,7 +606,7 @@ __global__ void fill_synth_kernel(void* dst, long n, uint64_t start, float offse
 cudaError_t fill_synth(void* dst, long n, uint64_t start, float offset, float c32, int bf16,
                        cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
-  fill_synth_kernel<<<grid_for(n, 256), 256, 0, s>>>(dst, n, start, offset, c32, bf16);
+  launch_kernel(fill_synth_kernel, grid_for(n, 256), 256, 0, s, dst, n, start, offset, c32, bf16);
   return cudaGetLastError();
 }
 

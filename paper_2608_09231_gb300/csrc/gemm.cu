@@ -79,6 +79,7 @@ template <typename T>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A, long lda,
                                                         const T* __restrict__ W, long ldw,
                                                         int M, int N, int K, const Epi e) {
+  grid_dep_sync();
   if (epi_skip(e.st, e.flag_want)) return;
   const int t = epi_step(e);
   __shared__ float As[16][64 + 4];
@@ -261,6 +262,7 @@ __global__ void __launch_bounds__(192, 1)
                    const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
                    const __grid_constant__ Epi e0, const __grid_constant__ Epi e1, int M0, int M1,
                    int N, int K, int a_split, int g0, int g1, int* err) {
+  grid_dep_sync();
   // Two independent problems with the same N and K may share one launch (problem 1 has
   // M1 rows, possibly 0): their tiles form one list, problem 0's first, so a small
   // problem fills the SMs the large one leaves idle in its last wave.
@@ -465,9 +467,9 @@ static cudaError_t launch_tc(const void* A0, long lda0, const void* W0, long ldw
   }
   const int tiles = ((M0 + TC_BM - 1) / TC_BM + (M1 + TC_BM - 1) / TC_BM) * (N / BN);
   const int grid = std::min(tiles, num_sms());
-  gemm_tc_kernel<BN><<<grid, 192, C::SMEM, s>>>(ta0, tb0, ta1, tb1, e0, e1, M0, M1, N, K, a_split,
-                                                tile_group_rows(M0, TC_BM, K, a_split),
-                                                tile_group_rows(M1, TC_BM, K, a_split), err);
+  launch_kernel(gemm_tc_kernel<BN>, grid, 192, C::SMEM, s, ta0, tb0, ta1, tb1, e0, e1, M0, M1, N, K,
+                a_split, tile_group_rows(M0, TC_BM, K, a_split),
+                tile_group_rows(M1, TC_BM, K, a_split), err);
   return cudaGetLastError();
 }
 
@@ -492,6 +494,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
                      const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
                      const __grid_constant__ Epi e0, const __grid_constant__ Epi e1, int M0, int M1,
                      int N, int K, int a_split, int g0, int g1, int* err) {
+  grid_dep_sync();
   // both CTAs of a pair see the same flag, so they leave together
   if (epi_skip(e0.st, e0.flag_want)) return;
   extern __shared__ uint8_t smem_raw[];
@@ -704,9 +707,9 @@ static cudaError_t launch_pair(const void* A0, long lda0, const void* W0, long l
     tb1 = tb0;
   }
   const int pairs = std::min(pair_tiles(M0, M1, N), num_sms() / 2);
-  gemm_pair_kernel<<<2 * pairs, 192, PR_SMEM, s>>>(ta0, tb0, ta1, tb1, e0, e1, M0, M1, N, K, a_split,
-                                                   tile_group_rows(M0, PR_BM, K, a_split),
-                                                   tile_group_rows(M1, PR_BM, K, a_split), err);
+  launch_kernel(gemm_pair_kernel, 2 * pairs, 192, PR_SMEM, s, ta0, tb0, ta1, tb1, e0, e1, M0, M1, N,
+                K, a_split, tile_group_rows(M0, PR_BM, K, a_split),
+                tile_group_rows(M1, PR_BM, K, a_split), err);
   return cudaGetLastError();
 }
 
@@ -797,12 +800,12 @@ cudaError_t gemm(const void* A, long lda, const void* W, long ldw, int M, int N,
   if (N % 4 != 0) return cudaErrorInvalidValue;
   dim3 grid((N + 63) / 64, (M + 63) / 64);
   if (in_bf16)
-    gemm_simt_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(
-        reinterpret_cast<const __nv_bfloat16*>(A), lda, reinterpret_cast<const __nv_bfloat16*>(W),
-        ldw, M, N, K, e);
+    launch_kernel(gemm_simt_kernel<__nv_bfloat16>, grid, 256, 0, s,
+                  reinterpret_cast<const __nv_bfloat16*>(A), lda,
+                  reinterpret_cast<const __nv_bfloat16*>(W), ldw, M, N, K, e);
   else
-    gemm_simt_kernel<float><<<grid, 256, 0, s>>>(reinterpret_cast<const float*>(A), lda,
-                                                 reinterpret_cast<const float*>(W), ldw, M, N, K, e);
+    launch_kernel(gemm_simt_kernel<float>, grid, 256, 0, s, reinterpret_cast<const float*>(A), lda,
+                  reinterpret_cast<const float*>(W), ldw, M, N, K, e);
   return cudaGetLastError();
 }
 

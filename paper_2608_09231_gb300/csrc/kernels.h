@@ -6,7 +6,30 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 namespace bag {
+
+// Set between consecutive kernels of one enqueued segment of a step: launch_kernel then
+// gives the launch programmatic stream serialization, so the kernel's CTAs are resident
+// and waiting (grid_dep_sync) when its predecessor completes.
+extern thread_local bool g_pdl;
+
+template <typename... P, typename... A>
+inline cudaError_t launch_kernel(void (*k)(P...), dim3 grid, dim3 block, size_t smem,
+                                 cudaStream_t s, A&&... args) {
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t c = {};
+  c.gridDim = grid;
+  c.blockDim = block;
+  c.dynamicSmemBytes = smem;
+  c.stream = s;
+  c.attrs = at;
+  c.numAttrs = g_pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&c, k, std::forward<A>(args)...);
+}
 
 // Per-sample state the step kernels read and write on the device, so that a whole
 // denoising step can be replayed from a CUDA graph with no host round trip.
