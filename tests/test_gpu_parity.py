@@ -575,3 +575,17 @@ def test_set_budget_between_samples(lib):
         ctx.set_budget(T + 1)
     assert ei.value.status == 1
     ctx.close()
+
+
+@pytest.mark.parametrize("name", ["flux_small", "wan_small"])
+def test_programmatic_launch_matches_stream_order(name, lib, monkeypatch):
+    """Programmatic dependent launch changes only when each kernel's CTAs are scheduled,
+    never what they compute: a sample with it (the default) and one with every kernel
+    in plain stream order give the same latent and schedule bit for bit."""
+    cfg = configs.get_config(name)
+    T, B = 6, 3
+    _, a, ma, la, na = _gpu_sample(cfg, T, B)
+    monkeypatch.setenv("BAG_PDL", "0")
+    _, b, mb, lb, nb = _gpu_sample(cfg, T, B)
+    assert na == nb == B and list(ma) == list(mb)
+    assert np.array_equal(a, b) and np.array_equal(la, lb)
