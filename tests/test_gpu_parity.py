@@ -205,7 +205,7 @@ def test_gemm_gelu_epilogue(M, N, K, lib):
     ctx.close()
 
 
-@pytest.mark.parametrize("rows,cols", [(37, 256), (1000, 3072), (5, 5120)])
+@pytest.mark.parametrize("rows,cols", [(37, 256), (1000, 3072), (5, 5120), (3655, 3072), (20000, 256)])
 def test_ln_mod_against_oracle(rows, cols, lib):
     ctx = bag.create("tiny", T=2, B=1)
     x = synth.normal(7, 1, rows * cols, 2.0).reshape(rows, cols) + 0.5
