@@ -34,7 +34,7 @@ ROPE_THETA = 10000.0
 LN_EPS = 1e-6
 
 _BASE = {
-    # configs[0]-style tiny stack: fp32 end to end, exhaustive parity
+    # tiny stack (2 single-stream blocks, d 256): fp32 end to end, exhaustive parity
     "tiny": dict(kind="single", hidden=256, heads=4, mlp=1024, n_double=0, n_single=2,
                  n_wan=0, grid=(1, 16, 16), n_txt=32, patch_ch=64, rope_axes=(0, 32, 32),
                  dtype="f32", weight_seed=0, gate_seed=100, T=10, budgets=(5,)),
