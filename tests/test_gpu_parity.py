@@ -246,6 +246,53 @@ def test_rel_l1_against_oracle(rows, cols, bf16, lib):
     ctx.close()
 
 
+def test_empty_inputs_are_no_ops_and_undefined_ones_are_rejected(lib):
+    """Zero rows (GEMM, LN-mod), zero queries (attention) and zero elements (residual
+    add) launch nothing and leave every output untouched; a relative L1 over no rows and
+    an attention over no keys have no value and are refused with EINVAL."""
+    ctx = bag.create("tiny", T=2, B=1)
+    bf = torch.bfloat16
+    C = torch.full((4, 64), 7.0, device="cuda")
+    ctx.gemm_bf16(torch.zeros((1, 64), dtype=bf, device="cuda"),
+                  torch.zeros((64, 64), dtype=bf, device="cuda"), None, C, 0, 64, 64)
+    x = torch.zeros((1, 256), device="cuda")
+    y = torch.full((1, 256), 7.0, dtype=bf, device="cuda")
+    ctx.ln_mod(x, torch.zeros(256, device="cuda"), torch.zeros(256, device="cuda"), y, 0, 256)
+    q = torch.zeros((1, 256), dtype=bf, device="cuda")
+    kv = torch.zeros((16, 256), dtype=bf, device="cuda")
+    o = torch.full((1, 256), 7.0, dtype=bf, device="cuda")
+    ctx.attention_bf16(q, kv, kv, o, 0, 16, 4, 64, 0, 1)
+    r = torch.full((8,), 7.0, device="cuda")
+    ctx.residual_add(r, torch.zeros(8, device="cuda"), torch.zeros(8, device="cuda"), 0)
+    torch.cuda.synchronize()
+    for t in (C, y, o, r):
+        assert bool(torch.all(t.float() == 7.0))
+    scratch = torch.empty(2, device="cuda")
+    out = torch.full((3,), 7.0, device="cuda")
+    with pytest.raises(bag.BagError) as ei:
+        ctx.rel_l1(x, x, 0, 256, scratch, out)
+    assert bag.STATUS[ei.value.status] == "BAG_EINVAL"
+    with pytest.raises(bag.BagError):
+        ctx.attention_bf16(q, kv, kv, o, 1, 0, 4, 64, 0, 1)
+    torch.cuda.synchronize()
+    assert bool(torch.all(out == 7.0)) and bool(torch.all(o.float() == 7.0))
+    ctx.close()
+
+
+@pytest.mark.parametrize("name", ["tiny", "flux_small"])
+def test_single_step_sample(name, lib):
+    """T = 1 (so B = 1): the one step is computed in full (Algorithm 2's forced first
+    step) and the sample is one uncached Euler step from sigma = 1 to 0."""
+    cfg = configs.get_config(name)
+    inp, out, m, log, nfe = _gpu_sample(cfg, 1, 1)
+    assert nfe == 1 and list(m) == [1]
+    W, g = synth.make_weights(cfg), synth.make_gate(cfg["gate_seed"])
+    ref = O.sample(cfg, W, g, inp, T=1, B=1)
+    rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
+    assert list(ref["mask"]) == [1]
+    assert float(np.max(np.abs(out - ref["x"]))) <= TOL[cfg["dtype"]] * rms
+
+
 def test_residual_add_exact(lib):
     ctx = bag.create("tiny", T=2, B=1)
     n = 1 << 20
@@ -258,8 +305,8 @@ def test_residual_add_exact(lib):
     ctx.close()
 
 
-# nq >= 1024 runs on the CTA-pair kernel (512 query rows per pair; ragged 1100 leaves
-# most of the last pair's rows empty; 77 keys are one masked key tile)
+# the tensor-core kernel takes 256 query rows per CTA (ragged 1100 and 129 leave most of
+# the last CTA's rows empty; 77 keys are one masked key tile)
 @pytest.mark.parametrize("nq,nk,heads,dh", [(300, 300, 2, 128), (129, 515, 3, 128),
                                             (288, 288, 4, 64), (4608, 4608, 1, 128),
                                             (1100, 700, 2, 128), (2048, 77, 3, 128)])

@@ -818,3 +818,107 @@ def test_unipc_sampler_budget_T_is_uncached_and_differs_from_euler():
     assert np.array_equal(a["x"], b["x"])
     e = O.sample(dict(cfg, sampler="euler"), W, g, inp, T=6, B=6)
     assert not np.allclose(a["x"], e["x"], atol=1e-6)
+
+
+# ---------------------------------------------------------------------------
+# the network's entry, exit and conditioning pieces
+# ---------------------------------------------------------------------------
+def test_token_positions_text_at_origin_then_image_row_major():
+    cfg = dict(grid=(2, 2, 3), n_txt=2, kind="mmdit")
+    pos = O.token_positions(cfg)
+    want = [(0, 0, 0)] * 2 + [(f, r, c) for f in range(2) for r in range(2) for c in range(3)]
+    assert pos.shape == (14, 3) and [tuple(int(v) for v in p) for p in pos] == want
+    wan = O.token_positions(dict(cfg, kind="wan"))  # Wan: no text rows in the sequence
+    assert [tuple(int(v) for v in p) for p in wan] == want[2:]
+
+
+def test_flow_lambda_closed_forms():
+    """lambda(sigma) = log((1 - sigma) / sigma): zero at sigma = 1/2, log 4 at 1/5,
+    odd under sigma -> 1 - sigma, decreasing, infinite at the ends."""
+    assert O.flow_lambda(0.5) == 0.0
+    assert abs(O.flow_lambda(0.2) - math.log(4.0)) < 1e-15
+    s = np.linspace(0.01, 0.99, 99)
+    lam = O.flow_lambda(s)
+    assert np.allclose(lam, -O.flow_lambda(1.0 - s), atol=1e-13)
+    assert np.all(np.diff(lam) < 0)
+    assert O.flow_lambda(1.0) == -np.inf and O.flow_lambda(0.0) == np.inf
+
+
+def test_patch_embed_selects_weight_columns():
+    """x W^T + b with W [d, C]: the unit input e_k gives column k of W plus the bias (a
+    transposed weight would give a row)."""
+    rng = np.random.default_rng(3)
+    C, d = 5, 7
+    G = {"pe_w": rng.normal(size=(d, C)), "pe_b": rng.normal(size=d)}
+    out = O.patch_embed(G, np.eye(C))
+    for k in range(C):
+        assert np.allclose(out[k], G["pe_w"][:, k] + G["pe_b"], atol=1e-15)
+
+
+def test_final_layer_shift_scale_order_and_brute_force():
+    """Final layer = Linear(LN-mod(h)) with (shift, scale) = SiLU(vec) W_f^T + b_f split
+    shift first.  Scale -1 removes h entirely (output = shift W^T + b), which fails if
+    the two halves were swapped; then a scalar-loop evaluation on a tiny case."""
+    rng = np.random.default_rng(4)
+    d, C, n = 6, 3, 4
+    h = rng.normal(size=(n, d)) * 2 + 1
+    shift = rng.normal(size=d)
+    G = {"fmod_w": np.zeros((2 * d, d)), "fmod_b": np.concatenate([shift, -np.ones(d)]),
+         "fin_w": rng.normal(size=(C, d)), "fin_b": rng.normal(size=C)}
+    out = O.final_layer(G, rng.normal(size=d), h)
+    assert np.allclose(out, np.broadcast_to(shift @ G["fin_w"].T + G["fin_b"], (n, C)), atol=1e-13)
+    G["fmod_w"] = rng.normal(size=(2 * d, d)) * 0.3
+    G["fmod_b"] = rng.normal(size=2 * d) * 0.3
+    vec = rng.normal(size=d)
+    sv = [v / (1.0 + math.exp(-v)) for v in vec]
+    mod = [sum(G["fmod_w"][o][j] * sv[j] for j in range(d)) + G["fmod_b"][o] for o in range(2 * d)]
+    out = O.final_layer(G, vec, h)
+    for r in range(n):
+        mu = sum(h[r]) / d
+        var = sum((h[r][j] - mu) ** 2 for j in range(d)) / d
+        y = [(1.0 + mod[d + j]) * (h[r][j] - mu) / math.sqrt(var + 1e-6) + mod[j] for j in range(d)]
+        for o in range(C):
+            want = sum(G["fin_w"][o][j] * y[j] for j in range(d)) + G["fin_b"][o]
+            assert abs(out[r][o] - want) < 1e-12
+
+
+def test_block_modulation_streams_and_wan_table():
+    """SiLU(0) = 0, so a zero conditioning vector leaves each projection's bias: the
+    single block's, the image and text streams' own (in that order), and for Wan the
+    shared projection's bias plus the block's table."""
+    rng = np.random.default_rng(5)
+    d = 4
+    z = np.zeros(d)
+    single = {"type": "single", "mod_w": rng.normal(size=(3 * d, d)), "mod_b": rng.normal(size=3 * d)}
+    assert np.array_equal(O.block_modulation({}, {}, single, z), single["mod_b"])
+    double = {"type": "double", "img_mod_w": rng.normal(size=(6 * d, d)), "img_mod_b": rng.normal(size=6 * d),
+              "txt_mod_w": rng.normal(size=(6 * d, d)), "txt_mod_b": rng.normal(size=6 * d)}
+    mi, mt = O.block_modulation({}, {}, double, z)
+    assert np.array_equal(mi, double["img_mod_b"]) and np.array_equal(mt, double["txt_mod_b"])
+    G = {"tproj_w": rng.normal(size=(6 * d, d)), "tproj_b": rng.normal(size=6 * d)}
+    wan = {"type": "wan", "mod_tab": rng.normal(size=6 * d)}
+    assert np.allclose(O.block_modulation({}, G, wan, z), G["tproj_b"] + wan["mod_tab"], atol=1e-15)
+    # away from zero the projection is W SiLU(vec) + b, W stored [out, in]
+    vec = rng.normal(size=d)
+    s = vec / (1.0 + np.exp(-vec))
+    assert np.allclose(O.block_modulation({}, {}, single, vec),
+                       [sum(single["mod_w"][o][j] * s[j] for j in range(d)) + single["mod_b"][o]
+                        for o in range(3 * d)], atol=1e-13)
+
+
+def test_first_modulated_input_reads_the_image_stream_modulation():
+    """The signal's observable is block 0's first LN-modulation of the image stream: with
+    a double block it takes the image stream's (shift, scale), not the text stream's."""
+    rng = np.random.default_rng(6)
+    d, n = 4, 5
+    blk = {"type": "double", "img_mod_w": np.zeros((6 * d, d)), "img_mod_b": rng.normal(size=6 * d),
+           "txt_mod_w": np.zeros((6 * d, d)), "txt_mod_b": rng.normal(size=6 * d)}
+    h = rng.normal(size=(n, d))
+    got = O.first_modulated_input({"hidden": d}, {}, [blk], rng.normal(size=d), h)
+    sh, sc = blk["img_mod_b"][:d], blk["img_mod_b"][d:2 * d]
+    for r in range(n):
+        mu = sum(h[r]) / d
+        var = sum((v - mu) ** 2 for v in h[r]) / d
+        for j in range(d):
+            want = (1.0 + sc[j]) * (h[r][j] - mu) / math.sqrt(var + 1e-6) + sh[j]
+            assert abs(got[r][j] - want) < 1e-12
