@@ -169,11 +169,14 @@ def _bf16_tensor(seed, shape, std=1.0):
     return v, torch.from_numpy(v).cuda().to(torch.bfloat16)
 
 
-# (4096, 3072, 3072), (1000, 19456, 192) and (4100, 4864, 320) have enough 256 x 256
-# tiles for the CTA-pair kernel (the last three with a ragged final row tile)
+# (4096, 3072, 3072), (1000, 19456, 192), (4100, 4864, 320) and (7000, 3072, 256) have
+# enough 256 x 256 tiles for the CTA-pair kernel (the last three with a ragged final row
+# tile); (50, 38912, 256) is one 128-row tile wide enough for the single-CTA 128 x 256
+# kernel on every SM (the shape of the per-sample modulation GEMM)
 @pytest.mark.parametrize("M,N,K", [(300, 256, 128), (129, 64, 64), (1000, 384, 512),
                                    (77, 512, 256), (4096, 3072, 3072), (50, 1024, 320),
-                                   (1000, 19456, 192), (4100, 4864, 320), (7000, 3072, 256)])
+                                   (1000, 19456, 192), (4100, 4864, 320), (7000, 3072, 256),
+                                   (50, 38912, 256)])
 @pytest.mark.parametrize("simt", [0, 1])
 def test_gemm_bf16_against_fp64(M, N, K, simt, lib):
     ctx = bag.create("tiny", T=2, B=1)
