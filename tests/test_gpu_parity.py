@@ -171,8 +171,8 @@ def _bf16_tensor(seed, shape, std=1.0):
 
 # (4096, 3072, 3072), (1000, 19456, 192), (4100, 4864, 320) and (7000, 3072, 256) have
 # enough 256 x 256 tiles for the CTA-pair kernel (the last three with a ragged final row
-# tile); (50, 38912, 256) is one 128-row tile wide enough for the single-CTA 128 x 256
-# kernel on every SM (the shape of the per-sample modulation GEMM)
+# tile); (50, 38912, 256) is less than one tile high and wide enough for the pair kernel
+# (the shape class of the per-sample modulation GEMM, M = T)
 @pytest.mark.parametrize("M,N,K", [(300, 256, 128), (129, 64, 64), (1000, 384, 512),
                                    (77, 512, 256), (4096, 3072, 3072), (50, 1024, 320),
                                    (1000, 19456, 192), (4100, 4864, 320), (7000, 3072, 256),
