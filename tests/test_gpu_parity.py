@@ -296,6 +296,42 @@ def test_single_step_sample(name, lib):
     assert float(np.max(np.abs(out - ref["x"]))) <= TOL[cfg["dtype"]] * rms
 
 
+def test_calls_out_of_state_are_refused_and_leave_the_context_usable(lib):
+    """ESTATE: a whole-sample call on a context whose sample is under way (or finished)
+    until bag_reset, and a block forward before bag_prepare; EORDER: a step past T.
+    After each refusal the context still samples, and equals a fresh context's sample."""
+    cfg = configs.get_config("tiny")
+    T, B = 3, 2
+    ctx = bag.create(cfg, T=T, B=B)
+    inp = synth.make_inputs(cfg)
+    x, txt, pooled = _dev_inputs(cfg, inp)
+    h = torch.zeros((cfg["n_txt"] + 256, cfg["hidden"]), device="cuda")
+    with pytest.raises(bag.BagError) as ei:
+        ctx.forward_block(0, 0, h)
+    assert bag.STATUS[ei.value.status] == "BAG_ESTATE"
+    x1 = x.clone()
+    ctx.step(x1, 0, txt, pooled, x1)
+    with pytest.raises(bag.BagError) as ei:
+        ctx.run(x1, txt, pooled)
+    assert bag.STATUS[ei.value.status] == "BAG_ESTATE"
+    for t in range(1, T):
+        ctx.step(x1, t, txt, pooled, x1)
+    with pytest.raises(bag.BagError) as ei:
+        ctx.step(x1, T, txt, pooled, x1)
+    assert bag.STATUS[ei.value.status] == "BAG_EORDER"
+    with pytest.raises(bag.BagError) as ei:
+        ctx.run(x1, txt, pooled)
+    assert bag.STATUS[ei.value.status] == "BAG_ESTATE"
+    ctx.reset()
+    x2 = x.clone()
+    m2, _, n2 = ctx.run(x2, txt, pooled)
+    torch.cuda.synchronize()
+    _, ref, mr, _, nr = _gpu_sample(cfg, T, B)
+    assert n2 == nr == B and list(m2) == list(mr)
+    assert np.array_equal(x2.cpu().numpy(), ref) and torch.equal(x1, x2)
+    ctx.close()
+
+
 def test_residual_add_exact(lib):
     ctx = bag.create("tiny", T=2, B=1)
     n = 1 << 20
