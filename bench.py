@@ -244,17 +244,43 @@ def dominant_roofline(recs, peaks, peak_src, cfg_name, f32=False):
             "share_of_profiled_time": g["ms"] / total}
 
 
+BLOCK_WORKLOADS = {
+    "flux": ("flux_block", {}, "FLUX-shaped single-stream block, 4096 img + 512 txt tokens, "
+             "d 3072, 24x128 heads, MLP 12288, bf16"),
+    "qwen": ("qwen", {"n_double": 1}, "Qwen-Image-shaped double-stream block, 6889 img + 256 "
+             "txt tokens, d 3072, 24x128 heads, MLP 12288, bf16"),
+    "wan": ("wan", {"n_wan": 1}, "Wan2.1-14B-shaped block (self-attention over 32760 tokens, "
+            "cross-attention to 512, FFN 13824), d 5120, 40x128 heads, bf16"),
+}
+
+
+def block_flops(cfg):
+    """Algorithmic flops of one block forward: its projections and attention."""
+    d, F, ni, nx = cfg["hidden"], cfg["mlp"], cfg["n_img"], cfg["n_txt"]
+    if cfg["kind"] == "wan":
+        return (2.0 * ni * d * 3 * d + 4.0 * ni * ni * d + 2.0 * ni * d * d          # self-attn
+                + 2.0 * ni * d * d + 2.0 * nx * d * 2 * d + 4.0 * ni * nx * d      # cross-attn
+                + 2.0 * ni * d * d + 4.0 * ni * d * F)                             # out, FFN
+    N = ni + nx
+    if cfg["n_double"] > 0:
+        return 2.0 * N * d * 3 * d + 4.0 * N * N * d + 2.0 * N * d * d + 4.0 * N * d * F
+    return 2.0 * N * d * (3 * d + F) + 2.0 * N * (d + F) * d + 4.0 * N * N * d
+
+
 def block_mode(args):
-    """One FLUX-shaped single-stream block forward (hidden 3072, 24 x 128 heads, MLP
-    12288, 4096 + 512 tokens) and the skip-path kernel: the per-block throughput of the
-    stack and the cost of a reused step.  Also the target of the ncu captures."""
+    """One block forward at a benchmark model's full width and token count (--config
+    flux: a FLUX single-stream block; qwen: a Qwen-Image double-stream block; wan: a
+    Wan2.1-14B block) and the skip-path kernel: the per-block throughput of the stack
+    and the cost of a reused step.  Also the target of the ncu captures."""
     import numpy as np
     import torch
 
     from paper_2608_09231_gb300 import bag, configs, synth
 
-    cfg = configs.get_config("flux_block", qk_norm=args.qk_norm)
-    d, F, N = cfg["hidden"], cfg["mlp"], cfg["n_img"] + cfg["n_txt"]
+    name, over, workload = BLOCK_WORKLOADS[args.config]
+    cfg = configs.get_config(name, qk_norm=args.qk_norm, **over)
+    d = cfg["hidden"]
+    N = cfg["n_img"] + (0 if cfg["kind"] == "wan" else cfg["n_txt"])
     ctx = bag.create(cfg, T=cfg["T"], B=1)
     stream = torch.cuda.current_stream()
     ctx.set_stream(stream.cuda_stream)
@@ -274,7 +300,7 @@ def block_mode(args):
     e1.record(stream)
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / args.steps
-    flops = 2.0 * N * d * (3 * d + F) + 2.0 * N * (d + F) * d + 4.0 * N * N * d
+    flops = block_flops(cfg)
     # skip path: h_out = h_in + R over the image stream
     n = cfg["n_img"] * d
     hin = h0[:cfg["n_img"]].contiguous()
@@ -292,9 +318,7 @@ def block_mode(args):
     peaks, src = _peaks()
     tf = flops / (ms * 1e-3) / 1e12
     gbs = 12.0 * n / (ms_skip * 1e-3) / 1e9
-    print(json.dumps({"mode": "block", "workload": "FLUX-shaped single-stream block, 4096 img + "
-                      "512 txt tokens, d 3072, 24x128 heads, MLP 12288, bf16"
-                      + (", QK-RMSNorm" if args.qk_norm else ""),
+    print(json.dumps({"mode": "block", "workload": workload + (", QK-RMSNorm" if args.qk_norm else ""),
                       "ms_per_block": ms, "block_tflops": tf,
                       "frac_of_bf16_burst": tf / peaks.get("bf16_tflops", 1900.0),
                       "skip_ms": ms_skip, "skip_gbs": gbs,
