@@ -547,6 +547,64 @@ def test_conditioning_closed_form():
     assert np.allclose(vec, G["t2_b"] + inp["pooled"])
 
 
+def _conditioning_loops(sigma, t1_w, t1_b, t2_w, t2_b, pooled):
+    """Scalar-loop conditioning vector: the 256-wide sinusoid of 1000 sigma (cos half,
+    then sin half, frequencies 10000^(-j/128)), a dense layer t1, SiLU, a dense layer t2
+    (weights stored [out][in]), plus the pooled text vector when one is given."""
+    tval = 1000.0 * sigma
+    e = [math.cos(tval * math.exp(-math.log(10000.0) * j / 128)) for j in range(128)]
+    e += [math.sin(tval * math.exp(-math.log(10000.0) * j / 128)) for j in range(128)]
+    h = []
+    for o in range(len(t1_b)):
+        acc = t1_b[o]
+        for i in range(256):
+            acc += t1_w[o][i] * e[i]
+        h.append(acc / (1.0 + math.exp(-acc)))
+    out = []
+    for o in range(len(t2_b)):
+        acc = t2_b[o]
+        for i in range(len(h)):
+            acc += t2_w[o][i] * h[i]
+        out.append(acc + (pooled[o] if pooled is not None else 0.0))
+    return out
+
+
+@pytest.mark.parametrize("kind", ["single", "wan"])
+def test_conditioning_brute_force(kind):
+    """The whole conditioning chain with non-zero weights against scalar loops; for the
+    Wan kind the pooled vector must not enter (time embedding only)."""
+    d = 8
+    rng = np.random.default_rng(7)
+    G = {"t1_w": rng.normal(0, 0.3, (d, 256)), "t1_b": rng.normal(0, 0.3, d),
+         "t2_w": rng.normal(0, 0.5, (d, d)), "t2_b": rng.normal(0, 0.3, d)}
+    pooled = rng.normal(0, 1, d)
+    cfg = {"kind": kind}
+    for sigma in (1.0, 0.37, 0.02):
+        got = O.conditioning(cfg, G, sigma, pooled)
+        want = _conditioning_loops(sigma, G["t1_w"].tolist(), G["t1_b"].tolist(),
+                                   G["t2_w"].tolist(), G["t2_b"].tolist(),
+                                   None if kind == "wan" else pooled.tolist())
+        assert np.allclose(got, want, rtol=1e-12, atol=1e-12), (kind, sigma)
+
+
+def test_conditioning_detects_plausible_mistakes():
+    """Dropping the SiLU, swapping the two layers' roles or transposing t1 each change the
+    vector by far more than rounding (the brute force above would catch them)."""
+    d = 8
+    rng = np.random.default_rng(11)
+    G = {"t1_w": rng.normal(0, 0.3, (d, 256)), "t1_b": rng.normal(0, 0.3, d),
+         "t2_w": rng.normal(0, 0.5, (d, d)), "t2_b": rng.normal(0, 0.3, d)}
+    pooled = rng.normal(0, 1, d)
+    cfg = {"kind": "single"}
+    got = np.array(O.conditioning(cfg, G, 0.6, pooled))
+    e = O.timestep_embedding(600.0)
+    no_silu = G["t2_w"] @ (G["t1_w"] @ e + G["t1_b"]) + G["t2_b"] + pooled
+    silu_after = O.silu(G["t2_w"] @ (G["t1_w"] @ e + G["t1_b"]) + G["t2_b"]) + pooled
+    no_pooled = got - pooled
+    for wrong in (no_silu, silu_after, no_pooled):
+        assert np.max(np.abs(got - wrong)) > 1e-3
+
+
 def test_drift_is_zero_when_nothing_moves_and_logged_features():
     """With the velocity forced to zero the latent never moves, so the first block's
     modulated input changes only through the time embedding; with that frozen too the
