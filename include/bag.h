@@ -143,13 +143,18 @@ bag_status bag_create(const bag_arch* arch, int T, int B, bag_ctx** out);
 /* Release every device resource of the context (null is a no-op). */
 void bag_destroy(bag_ctx* ctx);
 
-/* Text of the last error on this context (or of the last failed bag_create when ctx is
- * null).  Valid until the next call on the context. */
+/* Text of the last error on this context, or, when ctx is null, of the last failed
+ * context-free call (bag_create, bag_rel_l1_noalloc) made by the calling host thread
+ * (that text is kept per thread).  Valid until the next call on the context (ctx
+ * non-null) or the thread's next context-free call (ctx null). */
 const char* bag_last_error(bag_ctx* ctx);
 
 /* Order the context's work after, and before, the caller's `cuda_stream` (a
  * cudaStream_t; null = the legacy stream).  The context keeps its own stream for the
- * captured step graph and bridges the two with events on every call. */
+ * captured step graph and bridges the two with events on every call.  The paper runs
+ * the T decisions of a sample strictly in sequence (Sec. 3.1 problem setup,
+ * Algorithm 2); this call only chooses which caller stream that sequence is ordered
+ * against, it never reorders steps. */
 bag_status bag_set_stream(bag_ctx* ctx, void* cuda_stream);
 
 /* Replace the gate parameters (Eq. 1; App. A.2 z-scored inputs).  theta: host array of
@@ -173,7 +178,9 @@ bag_status bag_set_policy(bag_ctx* ctx, int policy, const uint8_t* host_mask, fl
  * between samples. */
 bag_status bag_set_budget(bag_ctx* ctx, int B);
 
-/* Start a new sample: t = 0, c = 0, cache invalid, sticky device error cleared. */
+/* Start a new sample (a new prompt): Algorithm 2's initial state, t = 0 and the spent
+ * budget c = 0, with the residual cache invalid so that step 0 computes (m_0 = 1,
+ * Sec. 3.1); the sticky device error is cleared. */
 bag_status bag_reset(bag_ctx* ctx);
 
 /* One sampler step (Algorithm 2, one iteration).  t must equal the context's next step
@@ -186,8 +193,11 @@ bag_status bag_step(bag_ctx* ctx, const float* x, int t, const bag_cond* cond, f
                     int32_t* full_or_cached);
 
 /* All T steps of one sample from the context's current state (normally right after
- * bag_reset), in place on x_inout (device fp32 [n_img, patch_ch]).  stats (optional,
- * host) receives the schedule after one synchronisation at the end. */
+ * bag_reset), in place on x_inout (device fp32 [n_img, patch_ch]): Algorithm 2's loop
+ * over t = 0 .. T-1, each iteration one bag_step (gate, pacing, full stack or cached
+ * residual, sampler update), with exactly B full evaluations (Sec. 3.2 budget-exact
+ * inference).  stats (optional, host) receives the schedule after one synchronisation
+ * at the end. */
 bag_status bag_run(bag_ctx* ctx, float* x_inout, const bag_cond* cond, bag_stats* stats);
 
 /* Same as bag_run with HOST buffers: copies x (fp32 [n_img, patch_ch]) and the
@@ -294,9 +304,11 @@ bag_status bag_rel_l1(bag_ctx* ctx, const void* a, const void* b, int dtype, lon
  * The row partials live in a fixed file-scope device array of 2 * 65536 floats held by
  * every GPU that loads the library until exit: rows > 65536 returns BAG_EINVAL.  The
  * first call on a device looks the array's address up (cudaGetSymbolAddress) and
- * should come before any stream capture.  All calls share the array and it keeps the
- * last call's contents (each call writes what it reads); calls that overlap on the GPU
- * race.  Errors are reported through bag_last_error(NULL). */
+ * should come before any stream capture; the address is kept per CUDA context and
+ * looked up again when the device's current context changes (e.g. after
+ * cudaDeviceReset).  All calls share the array and it keeps the last call's contents
+ * (each call writes what it reads); calls that overlap on the GPU race.  Errors are
+ * reported through bag_last_error(NULL). */
 bag_status bag_rel_l1_noalloc(const void* a, const void* b, int dtype, long rows, long cols,
                               float* out, void* cuda_stream);
 

@@ -106,8 +106,13 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t s);
 
 cudaError_t attention(const AttnArgs& a, int* err, cudaStream_t s, int force_simt) {
   if (a.nq <= 0) return cudaSuccess;
-  if (a.bf16 && !force_simt && attention_tc_supported(a)) return attention_tc(a, err, s);
-  // (until the tensor-core attention covers a shape, bf16 attention runs on CUDA cores)
+  // bf16 attention runs on the tensor cores; a call the tensor-core kernel cannot take
+  // (head_dim != 128, V not transposed, unaligned operands) is refused rather than sent
+  // to the CUDA-core kernel, which serves fp32 backbones and explicit cross-checks only
+  if (a.bf16 && !force_simt) {
+    if (!attention_tc_supported(a)) return cudaErrorNotSupported;
+    return attention_tc(a, err, s);
+  }
   dim3 grid((a.nq + 15) / 16, a.heads);
   if (a.dh == 64) {
     if (a.bf16)

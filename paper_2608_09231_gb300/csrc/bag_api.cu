@@ -179,7 +179,10 @@ struct bag_ctx {
   bool profiling = false;
 };
 
-static std::string g_create_error;
+// Errors of calls without a context (bag_create, bag_rel_l1_noalloc) are kept per host
+// thread, so that one thread's failure never overwrites or frees the text another thread
+// is reading through bag_last_error(NULL).
+static thread_local std::string g_create_error;
 thread_local bool bag::g_pdl = false;
 
 void bag::set_global_error(const std::string& msg) { g_create_error = msg; }
@@ -248,6 +251,8 @@ static bag_status validate_arch(const bag_arch* a, int T, int B) {
   if (a->kind == BAG_KIND_SINGLE && a->n_double) return fail(nullptr, BAG_EINVAL, "SINGLE kind has no double blocks");
   if (!(a->tau > 0.f && a->tau < 1.f)) return fail(nullptr, BAG_EINVAL, "tau must be in (0, 1)");
   if (a->dtype != BAG_F32 && a->dtype != BAG_BF16) return fail(nullptr, BAG_EINVAL, "dtype");
+  if (a->dtype == BAG_BF16 && dh != 128)
+    return fail(nullptr, BAG_EUNSUPPORTED, "bf16 backbones need head_dim 128 (tensor-core attention)");
   if (a->gate_kind < BAG_GATE_MLP3 || a->gate_kind > BAG_GATE_WAN6) return fail(nullptr, BAG_EINVAL, "gate_kind");
   if (a->cfg != 0 && a->cfg != 1) return fail(nullptr, BAG_EINVAL, "cfg must be 0 or 1");
   if (a->cfg && !std::isfinite(a->guidance)) return fail(nullptr, BAG_EINVAL, "guidance must be finite");

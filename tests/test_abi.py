@@ -90,6 +90,17 @@ def test_null_arguments(lib):
     lib.bag_destroy(None)
 
 
+def test_bf16_backbone_needs_tensor_core_head_dim(lib):
+    """bf16 attention runs only on the tensor-core kernel (head_dim 128); a bf16 backbone
+    with head_dim 64 is refused at creation instead of running on CUDA cores."""
+    a = bag.arch_from_config(configs.get_config("flux_small"))
+    a.heads = 8
+    a.rope_axes[:] = [16, 24, 24]
+    h = ctypes.c_void_p()
+    assert lib.bag_create(ctypes.byref(a), 4, 2, ctypes.byref(h)) == 7 and not h.value
+    assert "head_dim 128" in lib.bag_last_error(None).decode()
+
+
 def test_qk_norm_unsupported_for_wan(lib):
     st, h, msg = _create(lib, configs.get_config("wan_small"), 4, 2, qk_norm=1)
     assert st == 7 and not h.value and "qk_norm" in msg
