@@ -56,6 +56,12 @@ enum { BAG_GATE_MLP3 = 0, BAG_GATE_FLUX6 = 1, BAG_GATE_WAN6 = 2 };
  * B(h) = e^{-h} - 1, first order at the first and last step; the sampler the paper's Wan
  * experiments cache (Sec. 4.1).  Its multistep history lives in the context. */
 enum { BAG_SAMPLER_EULER = 0, BAG_SAMPLER_UNIPC = 1 };
+/* Observable of the trajectory signal (Eq. 3's drift and step change, relative L1).
+ * MODULATED: the first block's modulated input on the image stream (LayerNorm of the
+ * patch-embedded tokens under block 0's first adaLN shift and scale).  EMBEDDED: the
+ * post-patch-embedding token tensor x_t itself, the paper's observable (Eq. 3 and the
+ * paragraph after it; under guidance both branches share it). */
+enum { BAG_OBS_MODULATED = 0, BAG_OBS_EMBEDDED = 1 };
 enum {
   BAG_POLICY_BAG = 0,   /* Algorithm 2: gate decision + the two forced pacing rules */
   BAG_POLICY_FULL = 1,  /* uncached sampling: every step evaluates the network */
@@ -97,6 +103,7 @@ typedef struct {
                          and MMDIT kinds with BAG_BF16 only (else BAG_EUNSUPPORTED) */
   int sampler;        /* BAG_SAMPLER_* */
   float shift;        /* time shift s of the sigma grid (> 0; 0 is read as 1, no shift) */
+  int observable;     /* BAG_OBS_*: what the trajectory signal reads */
 } bag_arch;
 
 /* Conditioning of one sample (device pointers, read during bag_step / bag_run).
@@ -117,7 +124,7 @@ typedef struct {
  *   [0..2] (B-c)/B, (T-t)/T, drift;  [3] gate logit z;  [4] raw gate bit;  [5] m_t;
  *   [6] c before the step;  [7] t - t_last;  [8..10] B/T, (B-c)/B, (B-c)/(T-t);
  *   [11] sum|m_t - m_last|;  [12] sum|m_last|;  [13] step change;  [14] sum|m_t - m_{t-1}|;
- *   [15] sum|m_{t-1}|   (m = the first block's modulated image-stream input).
+ *   [15] sum|m_{t-1}|   (m = the signal's observable, see BAG_OBS_*).
  * nfe receives the realised number of full evaluations. */
 #define BAG_LOG_FLOATS 16
 typedef struct {
@@ -281,6 +288,14 @@ bag_status bag_gemm_bf16(bag_ctx* ctx, const void* A, long lda, const void* W, l
 bag_status bag_attention_bf16(bag_ctx* ctx, const void* q, const void* k, const void* v,
                               void* o, long ld, int nq, int nk, int heads, int dh, long vpad,
                               int force_simt);
+
+/* bag_attention_bf16 with fp16 q, k and v (same layouts; v transposed per head, vpad > 0)
+ * and a bf16 output o: the operand type the sampling path of bf16 backbones uses for
+ * attention (an 11-bit significand for q and k, whose rounding the softmax exponent
+ * amplifies; the softmax probabilities P enter the PV product as fp16 too).  Tensor-core
+ * kernel only (dh 128), else BAG_EUNSUPPORTED. */
+bag_status bag_attention_f16(bag_ctx* ctx, const void* q, const void* k, const void* v, void* o,
+                             long ld, int nq, int nk, int heads, int dh, long vpad);
 
 /* y = (1 + scale) * LayerNorm(x) + shift row-wise (eps 1e-6, no affine): x fp32 device
  * [rows, cols], shift/scale fp32 device [cols] (null = plain LayerNorm), y bf16 device. */

@@ -15,8 +15,10 @@ What it computes, and from which passage:
   * The gate z_t = g_theta(s_bud, s_traj) of Eq. 1, in the 3-input form the build
     targets (remaining-budget fraction, remaining-steps fraction, drift signal) with
     all six scalars of Eq. 3 logged beside it.
-  * The trajectory signal: relative L1 change of the first block's modulated input
-    against the last fully computed step (the drift entry of Eq. 3 with the L1 norm).
+  * The trajectory signal: relative L1 change of the observable against the last fully
+    computed step (the drift entry of Eq. 3 with the L1 norm); the observable is the
+    first block's modulated input by default, or the post-patch-embedding tokens, the
+    paper's own observable (Eq. 3), when cfg["observable"] == "embedded".
   * The DiT network evaluated at full steps: adaLN-modulated MMDiT blocks (modulated
     LayerNorm, QKV projection with RoPE, joint attention, output projection, GELU MLP,
     gated residuals).  The paper names the backbones (FLUX.1-dev, Qwen-Image, Wan2.1;
@@ -407,6 +409,16 @@ def patch_embed(G, x):
     return linear(x, G["pe_w"], G["pe_b"])
 
 
+def observable(cfg, G, blocks, vec, h_in):
+    """What the trajectory signal of Eq. 3 reads at a step.  'embedded': the
+    post-patch-embedding token tensor x_t itself, the paper's choice (Eq. 3 and the
+    paragraph after it; under guidance it is shared by both branches).  'modulated'
+    (default): the first block's modulated input on the image stream."""
+    if cfg.get("observable", "modulated") == "embedded":
+        return h_in
+    return first_modulated_input(cfg, G, blocks, vec, h_in)
+
+
 def run_stack(cfg, G, blocks, vec, h_img, txt):
     """Full network stack on the image stream h_img [N_i, d] with text txt; returns the
     image stream after the last block."""
@@ -680,7 +692,7 @@ def sample(cfg, W, gate, inputs, T, B, tau=0.5, policy="bag", drift_override=Non
     for t in range(T):
         vec = conditioning(cfg, G, sig[t], pooled)
         h_in = patch_embed(G, x)
-        m_t = first_modulated_input(cfg, G, blocks, vec, h_in)
+        m_t = observable(cfg, G, blocks, vec, h_in)
         rec = {"t": t, "c_before": c}
         if t == 0:
             full = 1

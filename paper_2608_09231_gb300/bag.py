@@ -20,6 +20,7 @@ KIND = {"single": 0, "mmdit": 1, "wan": 2}
 DTYPE = {"f32": 0, "bf16": 1}
 GATE_KIND = {"mlp3": 0, "flux6": 1, "wan6": 2}
 SAMPLER = {"euler": 0, "unipc": 1}
+OBSERVABLE = {"modulated": 0, "embedded": 1}
 POLICY_BAG, POLICY_FULL, POLICY_MASK, POLICY_STATIC_UNIFORM, POLICY_THRESHOLD = 0, 1, 2, 3, 4
 LOG_FLOATS = 16
 STATUS = {0: "BAG_OK", 1: "BAG_EINVAL", 2: "BAG_ENOMEM", 3: "BAG_ECUDA", 4: "BAG_EORDER",
@@ -28,7 +29,7 @@ STATUS = {0: "BAG_OK", 1: "BAG_EINVAL", 2: "BAG_ENOMEM", 3: "BAG_ECUDA", 4: "BAG
 EXPORTS = ["bag_create", "bag_destroy", "bag_last_error", "bag_set_stream", "bag_load_gate",
            "bag_set_policy", "bag_set_budget", "bag_reset", "bag_step", "bag_run", "bag_run_host",
            "bag_get_weight", "bag_forward_block", "bag_prepare", "bag_launch_count",
-           "bag_gemm_bf16", "bag_attention_bf16", "bag_ln_mod", "bag_residual_add",
+           "bag_gemm_bf16", "bag_attention_bf16", "bag_attention_f16", "bag_ln_mod", "bag_residual_add",
            "bag_profile_run", "bag_profile_launches", "bag_rel_l1", "bag_rel_l1_noalloc",
            "bag_check_wait_timeout"]
 
@@ -49,7 +50,8 @@ class Arch(ctypes.Structure):
                 ("dtype", ctypes.c_int), ("weight_seed", ctypes.c_uint64),
                 ("gate_seed", ctypes.c_uint64), ("tau", ctypes.c_float),
                 ("gate_kind", ctypes.c_int), ("cfg", ctypes.c_int), ("guidance", ctypes.c_float),
-                ("qk_norm", ctypes.c_int), ("sampler", ctypes.c_int), ("shift", ctypes.c_float)]
+                ("qk_norm", ctypes.c_int), ("sampler", ctypes.c_int), ("shift", ctypes.c_float),
+                ("observable", ctypes.c_int)]
 
 
 class Cond(ctypes.Structure):
@@ -108,6 +110,7 @@ def load(path=None):
         "bag_launch_count": ([_P, ctypes.POINTER(_L)], _I),
         "bag_gemm_bf16": ([_P, _P, _L, _P, _L, _P, _P, _L, _I, _I, _I, _I, _I], _I),
         "bag_attention_bf16": ([_P, _P, _P, _P, _P, _L, _I, _I, _I, _I, _L, _I], _I),
+        "bag_attention_f16": ([_P, _P, _P, _P, _P, _L, _I, _I, _I, _I, _L], _I),
         "bag_ln_mod": ([_P, _P, _P, _P, _P, _I, _I], _I),
         "bag_residual_add": ([_P, _P, _P, _P, _L], _I),
         "bag_rel_l1": ([_P, _P, _P, _I, _L, _L, _P, _P], _I),
@@ -142,6 +145,7 @@ def arch_from_config(cfg, tau=0.5):
     a.qk_norm = 1 if cfg.get("qk_norm") else 0
     a.sampler = SAMPLER[cfg.get("sampler", "euler")]
     a.shift = float(cfg.get("shift", 1.0))
+    a.observable = OBSERVABLE[cfg.get("observable", "modulated")]
     return a
 
 
@@ -292,6 +296,11 @@ class Context:
         """v: [nk, ld] when vpad == 0, else transposed per head [heads, dh, vpad]."""
         self._chk(self.lib.bag_attention_bf16(self.h, _ptr(q), _ptr(k), _ptr(v), _ptr(o),
                                               q.stride(0), nq, nk, heads, dh, vpad, force_simt))
+
+    def attention_f16(self, q, k, v, o, nq, nk, heads, dh, vpad):
+        """fp16 q, k and v (v transposed per head, [heads, dh, vpad]); bf16 output."""
+        self._chk(self.lib.bag_attention_f16(self.h, _ptr(q), _ptr(k), _ptr(v), _ptr(o),
+                                             q.stride(0), nq, nk, heads, dh, vpad))
 
     def ln_mod(self, x, shift, scale, y, rows, cols):
         self._chk(self.lib.bag_ln_mod(self.h, _ptr(x), _ptr(shift), _ptr(scale), _ptr(y), rows,

@@ -25,6 +25,9 @@ patch_ch    channels per image token in the latent (64 = 16-ch latent x 2x2 patc
 rope_axes   head-dim split of the rotary embedding over the (frame, row, col) axes
 dtype       'f32' or 'bf16' (GEMM / attention operand type)
 gate_kind   'mlp3' (3 inputs, default), 'flux6' or 'wan6' (the paper's six-input gates)
+observable  what the trajectory signal reads: 'modulated' (default; the first block's
+            modulated image-stream input) or 'embedded' (the post-patch-embedding
+            tokens, the paper's observable)
 """
 
 import copy
@@ -73,6 +76,19 @@ _SMALL = {
     "tiny_ragged": dict(_BASE["tiny"], grid=(1, 13, 11), n_txt=19, T=7, budgets=(3,)),
 }
 
+# Production width at reduced depth and token count: the blocks, head count, MLP width
+# and RoPE layout of the FLUX-, Qwen-Image- and Wan2.1-14B-shaped stacks, with one or
+# two blocks and 1000-1650 image tokens, so that the fp64 oracle runs a whole short
+# sample while every stack projection has enough 256 x 256 tiles (at least one per CTA
+# pair) to run on the CTA-pair GEMM.
+_WIDE = {
+    "flux_wide": dict(_BASE["flux"], n_double=1, n_single=1, grid=(1, 36, 36), n_txt=512,
+                      T=6, budgets=(3,)),
+    "qwen_wide": dict(_BASE["qwen"], n_double=1, grid=(1, 41, 40), n_txt=256, T=6,
+                      budgets=(3,)),
+    "wan_wide": dict(_BASE["wan"], n_wan=1, grid=(3, 16, 21), n_txt=512, T=6, budgets=(3,)),
+}
+
 
 def get_config(name, **overrides):
     """Return a fresh config dict with derived fields filled in."""
@@ -80,12 +96,15 @@ def get_config(name, **overrides):
         cfg = copy.deepcopy(_BASE[name])
     elif name in _SMALL:
         cfg = copy.deepcopy(_SMALL[name])
+    elif name in _WIDE:
+        cfg = copy.deepcopy(_WIDE[name])
     else:
         raise KeyError(f"unknown config {name!r}")
     cfg.update(overrides)
     cfg.setdefault("gate_kind", "mlp3")
     cfg.setdefault("sampler", "euler")     # "euler" or "unipc"
     cfg.setdefault("shift", 1.0)           # time shift of the sigma grid
+    cfg.setdefault("observable", "modulated")
     cfg["name"] = name
     d, h = cfg["hidden"], cfg["heads"]
     assert d % h == 0
@@ -99,4 +118,4 @@ def get_config(name, **overrides):
 
 
 def config_names():
-    return list(_BASE) + list(_SMALL)
+    return list(_BASE) + list(_SMALL) + list(_WIDE)

@@ -1,4 +1,4 @@
-// Joint attention on the 5th-generation tensor cores (head_dim 128, bf16 operands).
+// Joint attention on the 5th-generation tensor cores (head_dim 128, 16-bit operands).
 //
 // One CTA owns two 128-row query tiles (A and B) of one head and walks the keys in
 // tiles of 128:
@@ -9,7 +9,7 @@
 //               softmax runs
 //   warps 2..5  softmax of tile A, warps 6..9 softmax of tile B: thread = query row; S
 //               row read from TMEM into registers in one round trip, P = exp2(s - m)
-//               packed to bf16 and written back into TMEM over the S columns.
+//               packed to 16 bits and written back into TMEM over the S columns.
 // The PV product takes P straight from TMEM as its A operand, so P never touches
 // shared memory; shared memory only feeds Q, K and V^T.  O stays in TMEM for the whole
 // key loop.  The running max only moves (and O is rescaled in TMEM) when a tile's max
@@ -17,6 +17,10 @@
 // sum uses the same max, which makes the result the exact softmax up to rounding.
 // V arrives transposed per head ([head][dh][token]) from the QKV projection's epilogue,
 // which makes it a K-major B operand.
+// Operands are bf16 or fp16 (F16): q, k, v and P all of that type (an MMA's A and B share
+// one type).  The sampling path uses fp16: its 11-bit significand rounds q and k, whose
+// errors the softmax exponent amplifies, eight times more finely than bf16, and P stays
+// within fp16's range because the lazy maximum bounds it by 2^8.
 #include <cmath>
 
 #include "common.cuh"
@@ -117,6 +121,7 @@ BAG_DEV void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint3
 }
 }  // namespace
 
+template <bool F16>
 __global__ void __launch_bounds__(AT_THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, const AttnTcParams p) {
@@ -208,7 +213,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       // ---------------- MMA issuer ----------------
-      constexpr uint32_t idesc = idesc_bf16_f32(AT_M, AT_N);
+      constexpr uint32_t idesc = F16 ? idesc_f16_f32(AT_M, AT_N) : idesc_bf16_f32(AT_M, AT_N);
       const uint32_t q_addr = smem_u32(sQ);
       auto issue_s = [&](int x, int j) {
         const uint32_t qa = q_addr + x * AT_TILE;
@@ -318,7 +323,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         m_use = mx2;
         l *= alpha;
       }
-      // P = exp2(s * scale - m) (masked keys give exp2(-inf) = 0), packed bf16 pairs
+      // P = exp2(s * scale - m) (masked keys give exp2(-inf) = 0), packed 16-bit pairs
       // written over the S columns already read
       float ls0 = 0.f, ls1 = 0.f;
 #pragma unroll
@@ -331,7 +336,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
                p.scale_log2, -m_use);
           const float a0 = ex2(x0), a1 = ex2(x1);
           add2(ls0, ls1, a0, a1);
-          pk[i / 2] = pack_bf16x2(a0, a1);
+          pk[i / 2] = F16 ? pack_f16x2(a0, a1) : pack_bf16x2(a0, a1);
         }
         tmem_st16(s_addr + c * 16, pk);
       }
@@ -379,7 +384,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
 }
 
 cudaError_t attention_tc_init() {
-  return cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, AT_SMEM);
+  cudaError_t r = cudaFuncSetAttribute(attn_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       AT_SMEM);
+  if (r == cudaSuccess)
+    r = cudaFuncSetAttribute(attn_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, AT_SMEM);
+  return r;
 }
 
 int attention_tc_supported(const AttnArgs& a) {
@@ -408,7 +417,10 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t s) {
   p.flag_want = a.flag_want;
   p.err = err;
   dim3 grid((a.nq + 2 * AT_M - 1) / (2 * AT_M), a.heads);
-  launch_kernel(attn_tc_kernel, grid, AT_THREADS, AT_SMEM, s, tq, tk, tv, p);
+  if (a.f16)
+    launch_kernel(attn_tc_kernel<true>, grid, AT_THREADS, AT_SMEM, s, tq, tk, tv, p);
+  else
+    launch_kernel(attn_tc_kernel<false>, grid, AT_THREADS, AT_SMEM, s, tq, tk, tv, p);
   return cudaGetLastError();
 }
 

@@ -5,10 +5,12 @@
 //
 // One step, as enqueued (Algorithm 2, one iteration):
 //   prefix : patch embed  h_in = x W_pe^T + b  (also seeds the image stream)
-//            signal       m_t = LN-mod of h_in with block 0's first modulation, fused with
-//                         the per-row partial sums of |m_t - m_last| and |m_last|
+//            signal       m_t = LN-mod of h_in with block 0's first modulation (or h_in
+//                         itself, the paper's post-patch-embedding observable), fused
+//                         with the per-row partial sums of |m_t - m_last| and |m_last|;
+//                         after a full step it also takes m_last <- m_{t-1}
 //            gate         drift, gate MLP, forced rules, counters, log, decision
-//   full   : text tokens -> stream, every block, R = h_out - h_in, m_last <- m_t
+//   full   : text tokens -> stream, every block, R = h_out - h_in
 //   reuse  : h_out = h_in + R
 //   suffix : final LN-mod + projection fused with the Euler update, t += 1
 #include <algorithm>
@@ -262,6 +264,8 @@ static bag_status validate_arch(const bag_arch* a, int T, int B) {
   if (a->qk_norm && a->mlp % dh)
     return fail(nullptr, BAG_EUNSUPPORTED, "qk_norm needs mlp to be a multiple of head_dim");
   if (a->sampler != BAG_SAMPLER_EULER && a->sampler != BAG_SAMPLER_UNIPC) return fail(nullptr, BAG_EINVAL, "sampler");
+  if (a->observable != BAG_OBS_MODULATED && a->observable != BAG_OBS_EMBEDDED)
+    return fail(nullptr, BAG_EINVAL, "observable");
   if (!(a->shift == 0.f || (std::isfinite(a->shift) && a->shift > 0.f)))
     return fail(nullptr, BAG_EINVAL, "shift must be positive (0 = no shift)");
   return BAG_OK;
@@ -616,12 +620,16 @@ static bag_status alloc_activations(bag_ctx* ctx) {
   const long rows = wan ? ni : N;
   Arena A;
   A.add((void**)&ctx->x, (size_t)ni * ctx->C * 4);
-  A.add((void**)&ctx->xb, (size_t)ni * ctx->C * 2);
+  A.add((void**)&ctx->xb, (size_t)ni * ctx->C * 2 * 2);  // bf16 hi | lo halves of x
   A.add((void**)&ctx->h_in, (size_t)ni * d * 4);
   A.add((void**)&ctx->hj, (size_t)rows * d * 4);
   A.add((void**)&ctx->R, (size_t)ni * d * 4);
-  A.add(&ctx->m_cur, (size_t)ni * d * es);
-  A.add(&ctx->m_last, (size_t)ni * d * es);
+  // the signal's observable: in the operand precision for block 0's modulated input, in
+  // fp32 for the post-patch-embedding tokens (a small drift is a difference of two nearly
+  // equal tensors, which bf16 storage would bias)
+  const size_t obs_es = ctx->arch.observable == BAG_OBS_EMBEDDED ? 4 : es;
+  A.add(&ctx->m_cur, (size_t)ni * d * obs_es);
+  A.add(&ctx->m_last, (size_t)ni * d * obs_es);
   A.add((void**)&ctx->sig_partial, (size_t)ni * 4 * 4);
   A.add(&ctx->xn, (size_t)rows * d * es);
   A.add(&ctx->q, (size_t)rows * d * es);
@@ -752,6 +760,8 @@ static Epi base_epi(const bag_ctx* ctx, const DevState* st, int flag_want) {
   e.st = st;
   e.flag_want = flag_want;
   e.act_bf16 = ctx->act_bf16;
+  // attention operands of bf16 backbones are fp16 (see the attention kernel)
+  e.qkv_type = ctx->act_bf16 ? kStoreF16 : kStoreF32;
   return e;
 }
 
@@ -851,6 +861,7 @@ static void enq_attn(Enq& q, const void* Q, const void* K, const void* V, long v
   a.heads = ctx->H;
   a.dh = ctx->dh;
   a.bf16 = ctx->act_bf16;
+  a.f16 = ctx->act_bf16;  // q, k, v fp16 (written so by the projections' epilogues)
   a.st = st;
   a.flag_want = flag_want;
   q.pre(BAG_PROF_ATTN, 4.0 * nq * nk * ctx->H * ctx->dh,
@@ -988,7 +999,7 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int b
     e.kind = EPI_STORE;
     e.out = ctx->qc;
     e.ldo = d;
-    e.out_bf16 = ctx->act_bf16;
+    e.out_bf16 = ctx->act_bf16 ? kStoreF16 : kStoreF32;  // an attention operand
     e.bias = (const float*)blk.w.at("ca_q_b").p;
     enq_gemm(q, ctx->xn, d, blk.w.at("ca_q_w"), d, ni, (int)d, (int)d, e);
     Epi kv = base_epi(ctx, st, fw);
@@ -1051,9 +1062,19 @@ static void enq_prefix(Enq& q, int use_cond, unsigned long long handle) {
   pe.ldo = d;
   pe.out2 = img_stream(ctx);
   pe.ldo2 = d;
-  enq_gemm(q, ctx->act_bf16 ? (const void*)ctx->xb : (const void*)ctx->x, ctx->C, ctx->G.at("pe_w"),
-           ctx->C, ctx->ni, (int)d, ctx->C, pe);
-  // signal: block 0's first modulated input on the image stream (Eq. 3 drift)
+  if (ctx->act_bf16) {
+    // the latent enters as bf16 hi + lo halves (split A): the patch embedding, and with
+    // it the post-patch-embedding observable, carries no bf16 rounding of x
+    q.pre(BAG_PROF_GEMM, 4.0 * ctx->ni * d * ctx->C,
+          ((double)ctx->ni * 2 + d) * ctx->C * 2 + (double)ctx->ni * d * 8, ctx->ni, (int)d, 2 * ctx->C,
+          gemm_uses_pair(ctx->ni, 0, (int)d));
+    q.chk(gemm(ctx->xb, 2L * ctx->C, ctx->G.at("pe_w").p, ctx->C, ctx->ni, (int)d, ctx->C, 1, pe,
+               ctx->st ? &ctx->st->err : nullptr, q.s, 0, 1));
+  } else {
+    enq_gemm(q, ctx->x, ctx->C, ctx->G.at("pe_w"), ctx->C, ctx->ni, (int)d, ctx->C, pe);
+  }
+  // signal (Eq. 3 drift and step change) on the observable: block 0's first modulated
+  // input on the image stream, or the post-patch-embedding tokens themselves
   const Block& b0 = ctx->blocks[0];
   const float* m0 = ctx->mod_all + b0.mod_off;  // image-stream modulation comes first
   LnArgs a{};
@@ -1065,16 +1086,23 @@ static void enq_prefix(Enq& q, int use_cond, unsigned long long handle) {
   a.rows = ctx->ni;
   a.cols = (int)d;
   a.split = 0;
-  a.shift_a = a.shift_b = m0;
-  a.scale_a = a.scale_b = m0 + d;
+  if (ctx->arch.observable == BAG_OBS_EMBEDDED) {
+    a.identity = 1;
+    a.y_bf16 = 0;
+    a.shift_a = a.shift_b = a.scale_a = a.scale_b = nullptr;
+  } else {
+    a.shift_a = a.shift_b = m0;
+    a.scale_a = a.scale_b = m0 + d;
+  }
   a.mod_step = ctx->mod_stride;
   a.sig_ref = ctx->m_last;
-  a.sig_ref2 = ctx->m_cur;  // still the previous step's observable; replaced in place
+  a.sig_ref_w = ctx->m_last;  // refreshed here after a full step (m_last <- m_{t-1})
+  a.sig_ref2 = ctx->m_cur;    // still the previous step's observable; replaced in place
   a.sig_partial = ctx->sig_partial;
   a.sig_on = 1;
   a.st = ctx->st;
   a.flag_want = -1;
-  q.pre(BAG_PROF_SIGNAL, 0.0, (double)ctx->ni * d * (4.0 + 2.0 * ctx->act_size));
+  q.pre(BAG_PROF_SIGNAL, 0.0, (double)ctx->ni * d * (4.0 + 3.0 * (a.y_bf16 ? 2.0 : 4.0)));
   q.chk(ln_mod(a, q.s));
   q.pre(BAG_PROF_GATE, 0.0, (double)ctx->ni * 8);
   q.chk(gate_step(ctx->st, ctx->sig_partial, ctx->ni, ctx->d_gate, ctx->arch.gate_kind, ctx->thr, ctx->T, ctx->B,
@@ -1095,10 +1123,9 @@ static void enq_full(Enq& q, int fw) {
       q.chk(copy_rows_f32(ctx->st, fw, img_stream(ctx, br), d, ctx->h_in, d, 0, ctx->ni, (int)d, q.s));
     }
     for (int b = 0; b < ctx->nblk; ++b) enq_block(q, b, h, ctx->st, fw, br);
-    const long m_n = br ? 0 : (long)ctx->ni * d;
-    q.pre(BAG_PROF_CACHE, 0.0, (double)ctx->ni * d * 12.0 + (double)m_n * 2.0 * ctx->act_size);
-    q.chk(cache_refresh(ctx->st, img_stream(ctx, br), ctx->h_in, br ? ctx->R_u : ctx->R, ctx->m_last,
-                        ctx->m_cur, (long)ctx->ni * d, m_n, ctx->act_bf16, fw, q.s));
+    q.pre(BAG_PROF_CACHE, 0.0, (double)ctx->ni * d * 12.0);
+    q.chk(cache_refresh(ctx->st, img_stream(ctx, br), ctx->h_in, br ? ctx->R_u : ctx->R,
+                        (long)ctx->ni * d, fw, q.s));
   }
 }
 
@@ -1343,7 +1370,7 @@ static bag_status profile_run_impl(bag_ctx* ctx, float* x_inout, const bag_cond*
   std::vector<float> lg((size_t)ctx->T * kLogFloats);
   if (s == BAG_OK) {
     cudaMemcpyAsync(ctx->x, x_inout, xbytes, cudaMemcpyDeviceToDevice, ctx->stream);
-    if (ctx->act_bf16) to_bf16(ctx->xb, ctx->x, (long)ctx->ni * ctx->C, ctx->stream);
+    if (ctx->act_bf16) split_bf16(ctx->xb, ctx->x, ctx->ni, ctx->C, ctx->stream);
     for (int t = 0; t < ctx->T && s == BAG_OK; ++t) {
       long cnt = 0;
       Enq q{ctx, ctx->stream, &cnt};
@@ -1445,7 +1472,7 @@ static bag_status bag_step_impl(bag_ctx* ctx, const float* x, int t, const bag_c
   if (!ctx->prepared) return fail(ctx, BAG_ESTATE, "sample not prepared");
   const size_t xbytes = (size_t)ctx->ni * ctx->C * 4;
   CK(cudaMemcpyAsync(ctx->x, x, xbytes, cudaMemcpyDeviceToDevice, ctx->stream));
-  if (ctx->act_bf16) CK(to_bf16(ctx->xb, ctx->x, (long)ctx->ni * ctx->C, ctx->stream));
+  if (ctx->act_bf16) CK(split_bf16(ctx->xb, ctx->x, ctx->ni, ctx->C, ctx->stream));
   CKS(launch_step(ctx));
   CK(cudaMemcpyAsync(x_out, ctx->x, xbytes, cudaMemcpyDeviceToDevice, ctx->stream));
   if (full_or_cached)
@@ -1461,7 +1488,7 @@ static bag_status bag_run_impl(bag_ctx* ctx, float* x_inout, const bag_cond* con
   CKS(enq_prepare(ctx, cond));
   const size_t xbytes = (size_t)ctx->ni * ctx->C * 4;
   CK(cudaMemcpyAsync(ctx->x, x_inout, xbytes, cudaMemcpyDeviceToDevice, ctx->stream));
-  if (ctx->act_bf16) CK(to_bf16(ctx->xb, ctx->x, (long)ctx->ni * ctx->C, ctx->stream));
+  if (ctx->act_bf16) CK(split_bf16(ctx->xb, ctx->x, ctx->ni, ctx->C, ctx->stream));
   for (int t = 0; t < ctx->T; ++t) CKS(launch_step(ctx));
   CK(cudaMemcpyAsync(x_inout, ctx->x, xbytes, cudaMemcpyDeviceToDevice, ctx->stream));
   ctx->next_t = ctx->T;
@@ -1554,8 +1581,9 @@ static bag_status bag_gemm_bf16_impl(bag_ctx* ctx, const void* A, long lda, cons
   return BAG_OK;
 }
 
-static bag_status bag_attention_bf16_impl(bag_ctx* ctx, const void* q, const void* k, const void* v, void* o,
-                              long ld, int nq, int nk, int heads, int dh, long vpad, int force_simt) {
+static bag_status attention_op(bag_ctx* ctx, const void* q, const void* k, const void* v, void* o,
+                               long ld, int nq, int nk, int heads, int dh, long vpad, int force_simt,
+                               int f16) {
   if (!ctx || !q || !k || !v || !o) return BAG_EINVAL;
   if (nq < 0 || nk <= 0 || heads <= 0 || (dh != 64 && dh != 128) || ld < (long)heads * dh)
     return fail(ctx, BAG_EINVAL, "bad attention shape");
@@ -1576,8 +1604,10 @@ static bag_status bag_attention_bf16_impl(bag_ctx* ctx, const void* q, const voi
   a.heads = heads;
   a.dh = dh;
   a.bf16 = 1;
+  a.f16 = f16;
   a.st = nullptr;
   a.flag_want = -1;
+  if (f16 && force_simt) return fail(ctx, BAG_EUNSUPPORTED, "fp16 attention runs on the tensor cores only");
   if (!force_simt && !attention_tc_supported(a))
     return fail(ctx, BAG_EUNSUPPORTED, "tensor-core attention needs dh 128, transposed V and 16-byte alignment");
   CK(attention(a, &ctx->st_op->err, ctx->stream, force_simt));
@@ -1862,7 +1892,14 @@ bag_status bag_attention_bf16(bag_ctx* ctx, const void* q, const void* k, const 
                               long ld, int nq, int nk, int heads, int dh, long vpad, int force_simt) {
   if (!ctx) return BAG_EINVAL;
   CKS(enter(ctx));
-  return leave(ctx, bag_attention_bf16_impl(ctx, q, k, v, o, ld, nq, nk, heads, dh, vpad, force_simt));
+  return leave(ctx, attention_op(ctx, q, k, v, o, ld, nq, nk, heads, dh, vpad, force_simt, 0));
+}
+
+bag_status bag_attention_f16(bag_ctx* ctx, const void* q, const void* k, const void* v, void* o,
+                             long ld, int nq, int nk, int heads, int dh, long vpad) {
+  if (!ctx) return BAG_EINVAL;
+  CKS(enter(ctx));
+  return leave(ctx, attention_op(ctx, q, k, v, o, ld, nq, nk, heads, dh, vpad, 0, 1));
 }
 
 bag_status bag_ln_mod(bag_ctx* ctx, const float* x, const float* shift, const float* scale, void* y,

@@ -7,6 +7,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -52,6 +53,11 @@ BAG_DEV uint32_t pack_bf16x2(float a, float b) {
 }
 
 BAG_DEV float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+
+BAG_DEV uint32_t pack_f16x2(float a, float b) {
+  __half2 h = __floats2half2_rn(a, b);  // .x = a (low half), .y = b
+  return *reinterpret_cast<uint32_t*>(&h);
+}
 
 // ---------------------------------------------------------------------------
 // timers and bounded waits
@@ -253,6 +259,10 @@ BAG_DEV uint64_t sw128_desc(uint32_t saddr) {
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) |
          ((uint32_t)(M >> 4) << 24);
+}
+// Same with fp16 A and B operands (format field 0 for both)
+__host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N) {
+  return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
 BAG_DEV void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,

@@ -79,6 +79,16 @@ BAG_DEV void load4(const void* p, long off, int bf16, float* r) {
   }
 }
 
+// Four consecutive elements (16-bit or fp32) copied bit for bit.
+BAG_DEV void copy4(void* dst, const void* src, long off, int bf16) {
+  if (bf16)
+    *(reinterpret_cast<uint2*>(reinterpret_cast<__nv_bfloat16*>(dst) + off)) =
+        *(reinterpret_cast<const uint2*>(reinterpret_cast<const __nv_bfloat16*>(src) + off));
+  else
+    *(reinterpret_cast<float4*>(reinterpret_cast<float*>(dst) + off)) =
+        *(reinterpret_cast<const float4*>(reinterpret_cast<const float*>(src) + off));
+}
+
 // VPT float4 per thread (cols <= 128 * 4 * VPT): the row stays in registers, and the
 // smallest VPT that holds it keeps the register count low enough for many rows per SM
 // (the kernel is latency-bound at low occupancy).
@@ -102,17 +112,22 @@ __global__ void __launch_bounds__(LN_THREADS, VPT <= 6 ? 8 : (VPT <= 10 ? 5 : 4)
       s += (v[i].x + v[i].y) + (v[i].z + v[i].w);
     }
   }
-  const float mean = block_sum(s, red) / (float)a.cols;
-  float q = 0.f;
+  float mean = 0.f, rstd = 1.f;  // identity: y = x
+  if (!a.identity) {
+    mean = block_sum(s, red) / (float)a.cols;
+    float q = 0.f;
 #pragma unroll
-  for (int i = 0; i < VPT; ++i) {
-    const int c = threadIdx.x + i * LN_THREADS;
-    if (c < nv) {
-      const float dx = v[i].x - mean, dy = v[i].y - mean, dz = v[i].z - mean, dw = v[i].w - mean;
-      q += (dx * dx + dy * dy) + (dz * dz + dw * dw);
+    for (int i = 0; i < VPT; ++i) {
+      const int c = threadIdx.x + i * LN_THREADS;
+      if (c < nv) {
+        const float dx = v[i].x - mean, dy = v[i].y - mean, dz = v[i].z - mean, dw = v[i].w - mean;
+        q += (dx * dx + dy * dy) + (dz * dz + dw * dw);
+      }
     }
+    rstd = rsqrtf(block_sum(q, red) / (float)a.cols + 1e-6f);
   }
-  const float rstd = rsqrtf(block_sum(q, red) / (float)a.cols + 1e-6f);
+  // the previous step was fully computed: its observable (ref2) is the new reference
+  const bool refresh = a.sig_on && a.sig_ref_w && a.st && a.st->t > 0 && a.st->t_last == a.st->t - 1;
   const bool first = row < a.split;
   const float* sh = first ? a.shift_a : a.shift_b;
   const float* sc = first ? a.scale_a : a.scale_b;
@@ -144,8 +159,14 @@ __global__ void __launch_bounds__(LN_THREADS, VPT <= 6 ? 8 : (VPT <= 10 ? 5 : 4)
         // both references are read before y is stored: sig_ref2 may be the y buffer
         // itself (the previous step's observable, replaced by this step's)
         float r[4], r2[4], yy[4];
-        load4(a.sig_ref, off, a.y_bf16, r);
         load4(a.sig_ref2, off, a.y_bf16, r2);
+        if (refresh) {
+          copy4(a.sig_ref_w, a.sig_ref2, off, a.y_bf16);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) r[j] = r2[j];
+        } else {
+          load4(a.sig_ref, off, a.y_bf16, r);
+        }
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           yy[j] = a.y_bf16 ? bf16_round(y[j]) : y[j];
@@ -382,9 +403,9 @@ cudaError_t gate_step(DevState* st, const float* sig_partial, int sig_rows, cons
 // ---------------------------------------------------------------------------
 // residual cache
 // ---------------------------------------------------------------------------
+// (the drift reference m_last <- m_t is taken over by the next step's signal pass)
 __global__ void cache_refresh_kernel(const DevState* st, int flag_want, const float4* h_img,
-                                     const float4* h_in, float4* R, long n4, uint4* m_last,
-                                     const uint4* m_cur, long m16) {
+                                     const float4* h_in, float4* R, long n4) {
   grid_dep_sync();
   if (epi_skip(st, flag_want)) return;
   const long stride = (long)gridDim.x * blockDim.x;
@@ -392,7 +413,6 @@ __global__ void cache_refresh_kernel(const DevState* st, int flag_want, const fl
     const float4 a = h_img[i], b = h_in[i];
     R[i] = make_float4(a.x - b.x, a.y - b.y, a.z - b.z, a.w - b.w);
   }
-  for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < m16; i += stride) m_last[i] = m_cur[i];
 }
 
 __global__ void cache_reuse_kernel(const DevState* st, int flag_want, float4* h_img,
@@ -421,16 +441,12 @@ static int grid_for(long n, int threads) {
   return (int)b;
 }
 
-cudaError_t cache_refresh(const DevState* st, const float* h_img, const float* h_in, float* R,
-                          void* m_last, const void* m_cur, long n, long m_n, int m_bf16,
+cudaError_t cache_refresh(const DevState* st, const float* h_img, const float* h_in, float* R, long n,
                           int flag_want, cudaStream_t s) {
   if (n % 4 != 0) return cudaErrorInvalidValue;
-  const long mbytes = m_n * (m_bf16 ? 2 : 4);
-  if (mbytes % 16 != 0) return cudaErrorInvalidValue;
   launch_kernel(cache_refresh_kernel, grid_for(n / 4, 256), 256, 0, s, st, flag_want,
                 reinterpret_cast<const float4*>(h_img), reinterpret_cast<const float4*>(h_in),
-                reinterpret_cast<float4*>(R), n / 4, reinterpret_cast<uint4*>(m_last),
-                reinterpret_cast<const uint4*>(m_cur), mbytes / 16);
+                reinterpret_cast<float4*>(R), n / 4);
   return cudaGetLastError();
 }
 

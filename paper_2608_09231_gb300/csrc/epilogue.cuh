@@ -18,9 +18,28 @@ BAG_DEV bool epi_skip(const DevState* st, int flag_want) {
   return st != nullptr && flag_want >= 0 && st->flag != flag_want;
 }
 
+// type: kStoreF32, kStoreBF16 or kStoreF16
 template <int NV>
-BAG_DEV void store_vals(void* base, long idx, const float* v, int bf16) {
-  if (bf16) {
+BAG_DEV void store_vals(void* base, long idx, const float* v, int type) {
+  if (type == kStoreF16) {
+    __half* p = reinterpret_cast<__half*>(base) + idx;
+    if constexpr (NV % 8 == 0) {
+      if ((reinterpret_cast<uintptr_t>(p) & 15) == 0) {
+#pragma unroll
+        for (int j = 0; j < NV; j += 8) {
+          uint4 u;
+          u.x = pack_f16x2(v[j], v[j + 1]);
+          u.y = pack_f16x2(v[j + 2], v[j + 3]);
+          u.z = pack_f16x2(v[j + 4], v[j + 5]);
+          u.w = pack_f16x2(v[j + 6], v[j + 7]);
+          *reinterpret_cast<uint4*>(p + j) = u;
+        }
+        return;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < NV; ++j) p[j] = __float2half_rn(v[j]);
+  } else if (type == kStoreBF16) {
     __nv_bfloat16* p = reinterpret_cast<__nv_bfloat16*>(base) + idx;
     if constexpr (NV % 8 == 0) {
       if ((reinterpret_cast<uintptr_t>(p) & 15) == 0) {
@@ -152,14 +171,18 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float r
       const int cc = lc - region * e.d;
       if (region < 2) epi_qk_transform<NV>(e, jr, cc, region, v, rs);
       if (region == 0) {
-        store_vals<NV>(e.q, (long)jr * e.ldqk + cc, v, e.act_bf16);
+        store_vals<NV>(e.q, (long)jr * e.ldqk + cc, v, e.qkv_type);
       } else if (region == 1) {
-        store_vals<NV>(e.k, (long)jr * e.ldqk + cc, v, e.act_bf16);
+        store_vals<NV>(e.k, (long)jr * e.ldqk + cc, v, e.qkv_type);
       } else if (e.v_mode == 0) {
-        store_vals<NV>(e.v, (long)jr * e.ldqk + cc, v, e.act_bf16);
+        store_vals<NV>(e.v, (long)jr * e.ldqk + cc, v, e.qkv_type);
       } else {
         // transposed per head: vt[(head * dh + e) * vpad + token]
-        if (e.act_bf16) {
+        if (e.qkv_type == kStoreF16) {
+          __half* vt = reinterpret_cast<__half*>(e.v);
+#pragma unroll
+          for (int j = 0; j < NV; ++j) vt[(long)(cc + j) * e.vpad + jr] = __float2half_rn(v[j]);
+        } else if (e.qkv_type == kStoreBF16) {
           __nv_bfloat16* vt = reinterpret_cast<__nv_bfloat16*>(e.v);
 #pragma unroll
           for (int j = 0; j < NV; ++j) vt[(long)(cc + j) * e.vpad + jr] = __float2bfloat16_rn(v[j]);
@@ -237,7 +260,14 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float r
           x[j] = nx[j];
         }
       }
-      if (e.xb) store_vals<NV>(e.xb, (long)row * e.ldx + col0, nx, 1);
+      if (e.xb) {
+        // next step's patch-embedding operand: bf16 hi | lo halves of the new latent
+        float lo[NV];
+#pragma unroll
+        for (int j = 0; j < NV; ++j) lo[j] = nx[j] - bf16_round(nx[j]);
+        store_vals<NV>(e.xb, (long)row * 2 * e.ldx + col0, nx, kStoreBF16);
+        store_vals<NV>(e.xb, (long)row * 2 * e.ldx + e.ldx + col0, lo, kStoreBF16);
+      }
       break;
     }
     case EPI_VEC: {

@@ -157,7 +157,7 @@ static int tile_group_rows(int M, int BM, int K, int a_split) {
 constexpr int kVtScratchFloats = 32 * 33;
 constexpr int kVtScratchBytes = 4 * kVtScratchFloats * 4;  // four epilogue warps
 
-// V columns of a QKV projection with bf16 operands, stored transposed per head
+// V columns of a QKV projection with 16-bit (bf16 or fp16) storage, stored transposed per head
 // (vt[(head * dh + e) * vpad + token]): the warp's 32 rows x 32 columns pass through
 // shared memory, so each lane writes one column's 32 consecutive tokens as four 16-byte
 // stores instead of 32 two-byte stores.  Rows past M (the last tile) and token offsets
@@ -178,18 +178,22 @@ BAG_DEV void store_vt_warp(const Epi& e, int row, int col, float* v, float* sbuf
   const int row0 = row - lane;
   const int jr0 = row0 + e.row_off;
   const int cc = col + e.col_base - 2 * e.d + lane;  // this lane's column within V
-  __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(e.v) + (long)cc * e.vpad + jr0;
+  const bool f16 = e.qkv_type == kStoreF16;
+  uint16_t* dst = reinterpret_cast<uint16_t*>(e.v) + (long)cc * e.vpad + jr0;
   if (row0 + 31 < e.M && (jr0 & 7) == 0) {
     uint4 w[4];
     uint32_t* wp = reinterpret_cast<uint32_t*>(w);
 #pragma unroll
-    for (int k = 0; k < 16; ++k) wp[k] = pack_bf16x2(tc[2 * k], tc[2 * k + 1]);
+    for (int k = 0; k < 16; ++k)
+      wp[k] = f16 ? pack_f16x2(tc[2 * k], tc[2 * k + 1]) : pack_bf16x2(tc[2 * k], tc[2 * k + 1]);
 #pragma unroll
     for (int k = 0; k < 4; ++k) reinterpret_cast<uint4*>(dst)[k] = w[k];
   } else {
 #pragma unroll
     for (int k = 0; k < 32; ++k)
-      if (row0 + k < e.M) dst[k] = __float2bfloat16_rn(tc[k]);
+      if (row0 + k < e.M)
+        dst[k] = f16 ? __half_as_ushort(__float2half_rn(tc[k]))
+                     : __bfloat16_as_ushort(__float2bfloat16_rn(tc[k]));
   }
 }
 
@@ -197,7 +201,7 @@ BAG_DEV void store_vt_warp(const Epi& e, int row, int col, float* v, float* sbuf
 // the epilogue, columns col0 .. col0 + BN - 1.  vt_buf: this warp's transpose tile.
 template <int BN>
 BAG_DEV void drain_accumulator(const Epi& e, int t, int row, int col0, uint32_t tb, float* vt_buf) {
-  const bool vt_warp = e.kind == EPI_QKV && e.v_mode == 1 && e.act_bf16;
+  const bool vt_warp = e.kind == EPI_QKV && e.v_mode == 1 && e.qkv_type != kStoreF32;
   if (e.qn_q) {
     // QK-norm: the tile holds whole heads (BN a multiple of dh, checked at launch); a
     // first pass over each q / k head takes its sum of squares (bias included), the

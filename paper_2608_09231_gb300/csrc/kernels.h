@@ -3,6 +3,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -73,6 +74,9 @@ enum EpiKind : int {
 // sample, m_{i-1}, m_{i-2}, m_i; predictor weights of the corrected sample, m_i, m_{i-1}.
 enum { UC_SIG = 0, UC_CX, UC_CLAST, UC_CM1, UC_CM2, UC_CMT, UC_DX, UC_DM0, UC_DM1, kUniCoefs };
 
+// Storage types of epilogue outputs (the *_bf16 flags hold 0 or 1; type fields any)
+enum { kStoreF32 = 0, kStoreBF16 = 1, kStoreF16 = 2 };
+
 struct Epi {
   int kind = EPI_STORE;
   int M = 0, N = 0;
@@ -80,7 +84,7 @@ struct Epi {
   // plain stores
   void* out = nullptr;
   long ldo = 0;
-  int out_bf16 = 0;
+  int out_bf16 = 0;                // storage type of out (kStore*: 0 fp32, 1 bf16, 2 fp16)
   void* out2 = nullptr;
   long ldo2 = 0;
   int out2_bf16 = 0;
@@ -101,12 +105,13 @@ struct Epi {
   int row_off = 0;         // joint-sequence row of this GEMM's row 0
   int col_base = 0;        // logical column of this GEMM's column 0 (q=0, k=d, v=2d, mlp=3d)
   const float2* rope = nullptr;  // [joint rows][dh/2] (cos, sin); null = no rotation
-  int act_bf16 = 1;        // q/k/v/mlp storage type
+  int act_bf16 = 1;        // mlp storage type (1 bf16, 0 fp32)
+  int qkv_type = 1;        // q/k/v storage type (kStoreF32, kStoreBF16 or kStoreF16)
   void* mlp = nullptr;     // GELU(mlp) columns go to mlp[row * ldm + (col - 3d)]
   long ldm = 0;
   // sampler update
   float* x = nullptr;
-  __nv_bfloat16* xb = nullptr;
+  __nv_bfloat16* xb = nullptr;  // [rows, 2 * ldx]: bf16 hi | lo halves of the updated x
   long ldx = 0;
   const float* dsig = nullptr;  // [T]: sigma_{t+1} - sigma_t
   const float* qn_q = nullptr;  // EPI_QKV: per-head RMSNorm scales [dh] of q and k (both
@@ -153,7 +158,8 @@ struct AttnArgs {
   const void* v;  int v_mode; long ldv; long vpad;  // mode 0 like k; mode 1 [H][dh][vpad]
   void* o;        long ldo;      // output [Nq][ldo], head h at column h*dh
   int nq, nk, heads, dh;
-  int bf16;                      // operand/output type
+  int bf16;                      // 16-bit operands and output (else fp32)
+  int f16 = 0;                   // with bf16: q, k, v are fp16 (output stays bf16)
   const DevState* st; int flag_want;
 };
 cudaError_t attention(const AttnArgs& a, int* err, cudaStream_t s, int force_simt = 0);
@@ -170,8 +176,15 @@ struct LnArgs {
   const float* shift_b; const float* scale_b;
   long mod_step;
   // fused trajectory signal: per-row partial sums of |y - ref|, |ref|, |y - ref2|,
-  // |ref2| (4 floats per row); ref2 may alias y (it is read before y is stored)
+  // |ref2| (4 floats per row); ref2 may alias y (it is read before y is stored).
+  // sig_ref_w (optional, = sig_ref): when the previous step was fully computed
+  // (st->t_last == st->t - 1) its observable ref2 is the new reference, so the kernel
+  // reads ref2 once, takes it as ref and writes it into sig_ref_w as it goes (the
+  // reference refresh of Algorithm 2 without a separate copy).
   const void* sig_ref; const void* sig_ref2; float* sig_partial; int sig_on;
+  void* sig_ref_w = nullptr;
+  // identity: y = x (no normalisation or modulation; the observable is x itself)
+  int identity = 0;
   const DevState* st; int flag_want;
 };
 cudaError_t ln_mod(const LnArgs& a, cudaStream_t s);
@@ -180,8 +193,7 @@ cudaError_t gate_step(DevState* st, const float* sig_partial, int sig_rows, cons
                       int gate_kind, float thr, int T, int B, int policy,
                       const uint8_t* policy_mask, float delta, float* log,
                       unsigned long long cond_handle, int use_cond, cudaStream_t s);
-cudaError_t cache_refresh(const DevState* st, const float* h_img, const float* h_in, float* R,
-                          void* m_last, const void* m_cur, long n, long m_n, int m_bf16,
+cudaError_t cache_refresh(const DevState* st, const float* h_img, const float* h_in, float* R, long n,
                           int flag_want, cudaStream_t s);
 cudaError_t cache_reuse(const DevState* st, float* h_img, const float* h_in, const float* R,
                         long n, int flag_want, cudaStream_t s);

@@ -5,15 +5,16 @@ benchmark times.
   Wan2.1-14B) at full width and full token count, run through bag_forward_block,
   against the fp64 oracle evaluated one sampled row at a time (the oracle computes the
   keys and values of every token, and the block output only at the sampled rows).
-  Tolerance, derived from the arithmetic (bf16 operands, fp32 accumulation): a block
-  output is h + g * o, and o passes through at most four bf16 roundings of its operands
-  (LN-mod output, q/k/v or MLP hidden, P or GELU output, attention output), each a
-  relative error <= 2^-9.  Its error therefore scales with the element's own update
-  |g * o|, which at full width reaches ~5x the output RMS in columns with large adaLN
-  gates.  Bar per element: |err| <= 2e-2 x RMS(ref) + 2^-7 x |ref - h|.  Over the
-  sampled rows RMS(err) <= 2^-7 x RMS(ref - h): a Wan block adds three residual
-  branches (self-attention, cross-attention, FFN), each with its own roundings, and the
-  q and k roundings enter through the softmax exponent, where they count about double.
+  Tolerance, from the operand precision rather than from any kernel: a block output is
+  h + g * o, and o passes through the roundings of its operands (bf16 projection inputs,
+  fp16 q, k, v and P), each a relative error of at most 2^-8 (bf16) or 2^-11 (fp16), so
+  the error scales with the element's own update |g * o|, which at full width reaches
+  ~5x the output RMS in columns with large adaLN gates.  Bar per element:
+  |err| <= 2e-2 x RMS(ref) + 2^-7 x |ref - h|.  Over the sampled rows the error model of
+  tests/precision_model.py (the oracle evaluated with exactly those operand roundings)
+  predicts RMS(err) for the block; the GPU's RMS(err) must stay within 1.25x of it, so
+  the kernels add at most a quarter to the error their declared precision carries by
+  itself.  The text tokens enter both sides in bf16, as a bf16 context receives them.
 * Whole samples at full size: properties that hold at any size — realised NFE = B for
   every configured budget, m_0 = 1, the schedule equals Algorithm 2 applied to the gate
   bits the oracle computes from the GPU's logged gate inputs, and B = T reproduces
@@ -26,6 +27,7 @@ import torch
 
 from oracle import bag_oracle as O
 from paper_2608_09231_gb300 import bag, configs, synth
+from precision_model import bf16_inputs, operand_rounding
 
 pytestmark = pytest.mark.gpu
 
@@ -66,16 +68,24 @@ def test_block_full_size_sampled_rows(name, over, rows, lib):
     W = synth.make_weights(cfg, blocks=[0])
     G = O.to64(W)["global"]
     vec = O.conditioning(cfg, G, 1.0, inp["pooled"].astype(np.float64))
-    ref = O.forward_block(cfg, W, 0, h0.astype(np.float64), vec, rows=np.array(rows),
-                          txt=inp["txt"].astype(np.float64))
+    txt = bf16_inputs(inp)["txt"]
+    h64 = h0.astype(np.float64)
+    ref = O.forward_block(cfg, W, 0, h64, vec, rows=np.array(rows), txt=txt)
+    with operand_rounding(O):
+        model = O.forward_block(cfg, W, 0, h64, vec, rows=np.array(rows), txt=txt)
     rms = float(np.sqrt(np.mean(ref ** 2)))
     upd = ref - h0[rows]
     err = np.abs(got - ref)
+    rms_err, rms_model = float(np.sqrt(np.mean(err ** 2))), float(np.sqrt(np.mean((model - ref) ** 2)))
+    rms_upd = float(np.sqrt(np.mean(upd ** 2)))
+    print(f"{name} {over}: max|err| = {err.max():.4e} = {err.max() / rms:.3e} x RMS(ref) "
+          f"(model {np.max(np.abs(model - ref)) / rms:.3e}); RMS(err) / RMS(update) = "
+          f"{rms_err / rms_upd:.4e} (model {rms_model / rms_upd:.4e})")
     bar = 2e-2 * rms + 2.0 ** -7 * np.abs(upd)
     assert np.all(err <= bar), (float(err.max()), float((err / bar).max()))
-    assert float(np.sqrt(np.mean(err ** 2))) <= 2.0 ** -7 * float(np.sqrt(np.mean(upd ** 2)))
+    assert rms_err <= 1.25 * rms_model, (rms_err, rms_model)
     # the block changed the stream (it is not an identity pass)
-    assert float(np.sqrt(np.mean(upd ** 2))) > 100 * float(np.sqrt(np.mean(err ** 2)))
+    assert rms_upd > 100 * rms_err
 
 
 def _sample(ctx, cfg, inp):

@@ -375,6 +375,39 @@ def test_attention_against_oracle(nq, nk, heads, dh, simt, lib):
     ctx.close()
 
 
+@pytest.mark.parametrize("nq,nk,heads", [(300, 300, 2), (129, 515, 3), (4608, 4608, 1),
+                                         (1100, 700, 2), (2048, 77, 3)])
+def test_attention_f16_operands_against_oracle(nq, nk, heads, lib):
+    """The operand type the sampling path uses: fp16 q, k, v (and P), bf16 output.  With
+    11-bit operands the error is the output's bf16 rounding (<= 2^-8 relative) plus a small
+    share from the fp16 P and operand roundings."""
+    ctx = bag.create("tiny", T=2, B=1)
+    dh = 128
+    d = heads * dh
+
+    def f16(seed, shape):
+        v = synth.normal(seed, 77, int(np.prod(shape)), 1.0).reshape(shape).astype(np.float16)
+        return v.astype(np.float64), torch.from_numpy(v).cuda()
+
+    q, Q = f16(21, (nq, d))
+    k, K_ = f16(22, (nk, d))
+    v, V = f16(23, (nk, d))
+    o = torch.zeros((nq, d), dtype=torch.bfloat16, device="cuda")
+    vpad = (nk + 127) // 128 * 128
+    vt = torch.zeros((heads, dh, vpad), dtype=torch.float16, device="cuda")
+    vt[:, :, :nk] = V.reshape(nk, heads, dh).permute(1, 2, 0)
+    ctx.attention_f16(Q, K_, vt, o, nq, nk, heads, dh, vpad)
+    torch.cuda.synchronize()
+    rows = np.arange(nq) if nq <= 600 else np.r_[0:40, 250:290, 500:540, nq - 40:nq]
+    ref = O.attention(q.reshape(nq, heads, dh), k.reshape(nk, heads, dh),
+                      v.reshape(nk, heads, dh), q_rows=rows).reshape(len(rows), d)
+    got = o.float().cpu().numpy()[rows]
+    assert np.max(np.abs(got - ref)) <= 1.2 * 2.0 ** -8 * (np.max(np.abs(ref)) + 1e-3)
+    # elementwise: each output within its own bf16 rounding plus the fp16 share
+    assert np.all(np.abs(got - ref) <= 2.0 ** -8 * np.abs(ref) + 2.0 ** -10 * np.max(np.abs(ref)))
+    ctx.close()
+
+
 # ---------------------------------------------------------------------------
 # the paper's six-input gates (App. A.2) on all six scalars of Eq. 3
 # ---------------------------------------------------------------------------
@@ -401,6 +434,46 @@ def test_six_input_gate_sample_parity(name, kind, lib):
         assert abs(float(log[t, 13]) - sref) <= max(tol, 1e-6) * max(sref, 1e-3), t
     rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
     assert float(np.max(np.abs(got.astype(np.float64) - ref["x"]))) <= tol * rms
+
+
+@pytest.mark.parametrize("name,kind", [("flux_small", "flux6"), ("wan_small", "wan6"),
+                                       ("tiny_ragged", "mlp3"), ("qwen_small", "flux6")])
+def test_embedded_observable_sample_parity(name, kind, lib):
+    """The paper's observable (Eq. 3): the signal reads the post-patch-embedding tokens.
+    Schedules bit-exact on the GPU's logged gate inputs, the GPU's drift and step change
+    equal the oracle's own within the dtype's bar, and the latent within its bar."""
+    cfg = configs.get_config(name, gate_kind=kind, observable="embedded")
+    T, B = cfg["T"], cfg["budgets"][0]
+    inp, got, mask, log, nfe = _gpu_sample(cfg, T, B)
+    assert nfe == B and int(mask.sum()) == B and mask[0] == 1
+    g = synth.make_gate_any(cfg["gate_seed"], kind)
+    ref = O.sample(cfg, synth.make_weights(cfg), g, inp, T=T, B=B,
+                   drift_override=_gate_inputs(log),
+                   step_override=[None] + [float(v) for v in log[1:, 13]])
+    assert list(mask) == ref["mask"]
+    # fp32 observable from a split-precision patch embedding: the drift carries only fp32
+    # rounding (the latent itself differs by the dtype's bar, so allow that share)
+    tol = max(TOL[cfg["dtype"]], 1e-6)
+    for t in range(1, T):
+        dref, sref = ref["log"][t]["drift"], ref["log"][t]["s_traj"][2]
+        assert abs(float(log[t, 2]) - dref) <= tol * max(dref, 1e-3), t
+        assert abs(float(log[t, 13]) - sref) <= tol * max(sref, 1e-3), t
+        if kind == "mlp3":
+            assert O.gate_logit([np.float32(v) for v in log[t, 0:3]], g) == np.float32(log[t, 3])
+        else:
+            f = O.gate_features6(B, T, int(log[t, 6]), t, t - int(log[t, 7]), float(log[t, 2]),
+                                 float(log[t, 13]))
+            assert O.gate_logit6(f, g) == np.float32(log[t, 3]), t
+    rms = float(np.sqrt(np.mean(ref["x"] ** 2)))
+    assert float(np.max(np.abs(got.astype(np.float64) - ref["x"]))) <= TOL[cfg["dtype"]] * rms
+    # the GPU read the embedded observable: on the same schedule its drifts are closer to
+    # the oracle's embedded drifts than to the drifts of the default (modulated) observable
+    mod = O.sample(configs.get_config(name, gate_kind=kind), synth.make_weights(cfg), g, inp,
+                   T=T, B=B, policy=ref["mask"])
+    gpu = np.array([float(v) for v in log[1:, 2]])
+    emb = np.array([ref["log"][t]["drift"] for t in range(1, T)])
+    other = np.array([mod["log"][t]["drift"] for t in range(1, T)])
+    assert np.sum(np.abs(gpu - emb)) < 0.1 * np.sum(np.abs(gpu - other))
 
 
 @pytest.mark.parametrize("kind,n", [("mlp3", 81), ("flux6", 449), ("wan6", 785)])

@@ -605,6 +605,55 @@ def test_conditioning_detects_plausible_mistakes():
         assert np.max(np.abs(got - wrong)) > 1e-3
 
 
+def test_embedded_observable_closed_form_on_constant_velocity_net():
+    """The paper's observable (Eq. 3): the post-patch-embedding tokens.  With the final
+    layer's weight zeroed the velocity is the constant bias b at every step, so
+    x_t = x_0 + (sigma_t - 1) b and every row of h_t - h_s equals
+    (sigma_t - sigma_s) W_pe b: the drift and the step change have closed forms."""
+    cfg, W, g, inp = _tiny(grid=(1, 6, 6), n_txt=5, observable="embedded")
+    W["global"]["fin_w"][:] = 0.0
+    T, B = 8, 4
+    r = O.sample(cfg, W, g, inp, T=T, B=B)
+    G = O.to64(W)["global"]
+    sig = O.sigma_grid(T)
+    b = G["fin_b"]
+    x0 = inp["x"].astype(np.float64)
+    u = G["pe_w"] @ b
+    n = x0.shape[0]
+
+    def h(t):
+        return (x0 + (sig[t] - 1.0) * b) @ G["pe_w"].T + G["pe_b"]
+
+    last = 0
+    for t in range(1, T):
+        drift = n * abs(sig[t] - sig[last]) * np.abs(u).sum() / np.abs(h(last)).sum()
+        step = n * abs(sig[t] - sig[t - 1]) * np.abs(u).sum() / np.abs(h(t - 1)).sum()
+        rec = r["log"][t]
+        assert abs(rec["drift"] - drift) <= 1e-12 * max(1.0, drift), t
+        assert abs(rec["s_traj"][2] - step) <= 1e-12 * max(1.0, step), t
+        assert rec["s_traj"][0] == t - last
+        if r["mask"][t]:
+            last = t
+    # the default observable (block 0's modulated input) reads something else
+    r2 = O.sample(dict(cfg, observable="modulated"), W, g, inp, T=T, B=B, policy=r["mask"])
+    assert abs(r2["log"][1]["drift"] - r["log"][1]["drift"]) > 1e-6
+
+
+def test_observable_selects_the_embedded_tokens_or_the_modulated_input():
+    """At one step the embedded observable is the patch-embedded tensor itself, whatever
+    the blocks hold; the default is the first block's LayerNorm-modulated image stream."""
+    cfg, W, g, inp = _tiny(grid=(1, 6, 6), n_txt=5)
+    W64 = O.to64(W)
+    G, blocks = W64["global"], W64["blocks"]
+    vec = O.conditioning(cfg, G, 0.7, inp["pooled"].astype(np.float64))
+    h = O.patch_embed(G, inp["x"].astype(np.float64))
+    emb = O.observable(dict(cfg, observable="embedded"), G, blocks, vec, h)
+    assert emb is h
+    mod = O.observable(cfg, G, blocks, vec, h)
+    assert np.array_equal(mod, O.first_modulated_input(cfg, G, blocks, vec, h))
+    assert np.max(np.abs(mod - h)) > 0.1
+
+
 def test_drift_is_zero_when_nothing_moves_and_logged_features():
     """With the velocity forced to zero the latent never moves, so the first block's
     modulated input changes only through the time embedding; with that frozen too the
