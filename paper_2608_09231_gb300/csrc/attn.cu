@@ -94,10 +94,11 @@ __global__ void __launch_bounds__(128) attn_simt_kernel(const AttnArgs a) {
     for (int r = 0; r < R; ++r) {
       const long idx = (long)q * a.ldo + head * DH + lane + 32 * r;
       const float val = o[qi][r] * inv;
+      void* ob = (a.o2 && q >= a.o_split) ? a.o2 : a.o;
       if (a.bf16)
-        reinterpret_cast<__nv_bfloat16*>(a.o)[idx] = __float2bfloat16_rn(val);
+        reinterpret_cast<__nv_bfloat16*>(ob)[idx] = __float2bfloat16_rn(val);
       else
-        reinterpret_cast<float*>(a.o)[idx] = val;
+        reinterpret_cast<float*>(ob)[idx] = val;
     }
   }
 }

@@ -45,6 +45,8 @@ struct AttnTcParams {
   int nq, nk;
   void* o;
   long ldo;
+  void* o2;     // rows >= o_split are written to o2 (same row index and stride)
+  int o_split;
   float scale_log2;
   const DevState* st;
   int flag_want;
@@ -363,7 +365,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         tc_fence_after();
         const float inv = 1.f / l;
         const int q = q0 + x * AT_M + row;
-        __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.o) + (long)q * p.ldo + head * AT_D;
+        void* ob = (p.o2 && q >= p.o_split) ? p.o2 : p.o;
+        __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(ob) + (long)q * p.ldo + head * AT_D;
 #pragma unroll 1
         for (int c = 0; c < AT_D / 32; ++c) {
           float o[32];
@@ -412,6 +415,8 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t s) {
   p.nk = a.nk;
   p.o = a.o;
   p.ldo = a.ldo;
+  p.o2 = a.o2;
+  p.o_split = a.o_split;
   p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)AT_D));
   p.st = a.st;
   p.flag_want = a.flag_want;

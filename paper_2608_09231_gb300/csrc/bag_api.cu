@@ -146,7 +146,7 @@ struct bag_ctx {
   // classifier-free guidance: the unconditional branch's stream, cached residual, staged
   // conditioning and modulation (Wan: mod_all_u aliases mod_all, its modulation does not
   // depend on the text), and the conditional velocity of the current step
-  float *hj_u = nullptr, *R_u = nullptr, *vcond = nullptr;
+  float *R_u = nullptr, *vcond = nullptr;
   void* txt_stage_u = nullptr;
   float *pooled_stage_u = nullptr, *vec_all_u = nullptr, *svec_u = nullptr, *mod_all_u = nullptr;
   DevState* st = nullptr;     // sampler state
@@ -617,7 +617,10 @@ static bag_status alloc_activations(bag_ctx* ctx) {
   const bool wan = ctx->arch.kind == BAG_KIND_WAN;
   ctx->vpad = ((long)ctx->nrope + 127) / 128 * 128;
   ctx->vpad_c = ((long)nx + 127) / 128 * 128;
-  const long rows = wan ? ni : N;
+  // under guidance both branches share one stream and one set of activation buffers
+  // (rows of both branches, see enq_block)
+  const long nb = ctx->arch.cfg ? 2 : 1;
+  const long rows = (wan ? ni : N) * nb;
   Arena A;
   A.add((void**)&ctx->x, (size_t)ni * ctx->C * 4);
   A.add((void**)&ctx->xb, (size_t)ni * ctx->C * 2 * 2);  // bf16 hi | lo halves of x
@@ -634,14 +637,14 @@ static bag_status alloc_activations(bag_ctx* ctx) {
   A.add(&ctx->xn, (size_t)rows * d * es);
   A.add(&ctx->q, (size_t)rows * d * es);
   A.add(&ctx->k, (size_t)rows * d * es);
-  A.add(&ctx->vt, std::max((size_t)rows * d, (size_t)d * ctx->vpad) * es);
+  A.add(&ctx->vt, std::max((size_t)rows * d, (size_t)nb * d * ctx->vpad) * es);
   A.add(&ctx->cat, (size_t)rows * (d + F) * es);
   if (wan) {
-    A.add(&ctx->qc, (size_t)ni * d * es);
-    A.add(&ctx->kc, (size_t)nx * d * es);
-    A.add(&ctx->vtc, std::max((size_t)nx * d, (size_t)d * ctx->vpad_c) * es);
+    A.add(&ctx->qc, (size_t)nb * ni * d * es);
+    A.add(&ctx->kc, (size_t)nb * nx * d * es);
+    A.add(&ctx->vtc, std::max((size_t)nb * nx * d, (size_t)nb * d * ctx->vpad_c) * es);
   }
-  A.add(&ctx->txt_stage, (size_t)nx * d * es);
+  A.add(&ctx->txt_stage, (size_t)nb * nx * d * es);  // [text_c; text_u]
   A.add((void**)&ctx->pooled_stage, (size_t)d * 4);
   A.add((void**)&ctx->rope, (size_t)ctx->nrope * (ctx->dh / 2) * sizeof(float2));
   A.add((void**)&ctx->dsig, (size_t)T * 4);
@@ -660,10 +663,8 @@ static bag_status alloc_activations(bag_ctx* ctx) {
   A.add((void**)&ctx->mod_all, (size_t)T * ctx->mod_stride * 4);
   if (wan) A.add((void**)&ctx->wan_shared, (size_t)T * 8 * d * 4);
   if (ctx->arch.cfg) {
-    A.add((void**)&ctx->hj_u, (size_t)rows * d * 4);
     A.add((void**)&ctx->R_u, (size_t)ni * d * 4);
     A.add((void**)&ctx->vcond, (size_t)ni * ctx->C * 4);
-    A.add(&ctx->txt_stage_u, (size_t)nx * d * es);
     if (!wan) {
       A.add((void**)&ctx->pooled_stage_u, (size_t)d * 4);
       A.add((void**)&ctx->vec_all_u, (size_t)T * d * 4);
@@ -681,6 +682,7 @@ static bag_status alloc_activations(bag_ctx* ctx) {
   if (cudaMalloc(&ctx->aarena, A.off) != cudaSuccess)
     return fail(ctx, BAG_ENOMEM, "activation allocation of " + std::to_string(A.off) + " bytes failed");
   A.bind((char*)ctx->aarena);
+  if (ctx->arch.cfg) ctx->txt_stage_u = (char*)ctx->txt_stage + (size_t)nx * d * es;
   if (ctx->arch.cfg && wan) ctx->mod_all_u = ctx->mod_all;
   CK(cudaMemset(ctx->aarena, 0, A.off));
   std::vector<float2> tab;
@@ -825,6 +827,38 @@ static void enq_ln(Enq& q, const float* x, long ldx, void* y, long ldy, int rows
   q.chk(ln_mod(a, q.s));
 }
 
+// LayerNorm + modulation with four row segments [0, s1), [s1, s2), [s2, s3), [s3, rows),
+// each under its own modulation (shift at m, scale at m + d).
+static void enq_ln4(Enq& q, const float* x, long ldx, void* y, long ldy, int rows, int s1, int s2, int s3,
+                    const float* ma, const float* mb, const float* mc, const float* md, const DevState* st,
+                    int flag_want) {
+  const long d = q.ctx->d;
+  LnArgs a{};
+  a.x = x;
+  a.ldx = ldx;
+  a.y = y;
+  a.ldy = ldy;
+  a.y_bf16 = q.ctx->act_bf16;
+  a.rows = rows;
+  a.cols = (int)d;
+  a.split = s1;
+  a.split2 = s2;
+  a.split3 = s3;
+  a.shift_a = ma;
+  a.scale_a = ma + d;
+  a.shift_b = mb;
+  a.scale_b = mb + d;
+  a.shift_c = mc;
+  a.scale_c = mc + d;
+  a.shift_d = md;
+  a.scale_d = md + d;
+  a.mod_step = q.ctx->mod_stride;
+  a.st = st;
+  a.flag_want = flag_want;
+  q.pre(BAG_PROF_NORM, 0.0, (double)rows * d * (4.0 + q.ctx->act_size));
+  q.chk(ln_mod(a, q.s));
+}
+
 static void enq_qkv_epi(const bag_ctx* ctx, Epi& e, int row_off, bool rope) {
   e.kind = EPI_QKV;
   e.q = ctx->q;
@@ -843,7 +877,8 @@ static void enq_qkv_epi(const bag_ctx* ctx, Epi& e, int row_off, bool rope) {
 }
 
 static void enq_attn(Enq& q, const void* Q, const void* K, const void* V, long vpad, void* O,
-                     long ldo, int nq, int nk, const DevState* st, int flag_want) {
+                     long ldo, int nq, int nk, const DevState* st, int flag_want,
+                     void* O2 = nullptr, int o_split = 0) {
   const bag_ctx* ctx = q.ctx;
   AttnArgs a{};
   a.q = Q;
@@ -856,6 +891,8 @@ static void enq_attn(Enq& q, const void* Q, const void* K, const void* V, long v
   a.vpad = vpad;
   a.o = O;
   a.ldo = ldo;
+  a.o2 = O2;
+  a.o_split = o_split;
   a.nq = nq;
   a.nk = nk;
   a.heads = ctx->H;
@@ -869,22 +906,38 @@ static void enq_attn(Enq& q, const void* Q, const void* K, const void* V, long v
   q.chk(attention(a, ctx->st ? &ctx->st->err : nullptr, q.s));
 }
 
-// Per-branch buffers: br 0 is the conditional (or only) branch, br 1 the unconditional
-// branch of classifier-free guidance.
-static float* br_stream(const bag_ctx* ctx, int br) { return br ? ctx->hj_u : ctx->hj; }
+// Per-branch buffers: branch 0 is the conditional (or only) branch, branch 1 the
+// unconditional branch of classifier-free guidance.  Under guidance both branches live
+// in one stream, ordered [text_c; text_u; image_c; image_u] (Wan: [image_c; image_u]),
+// so that every projection takes both branches' rows in one launch; the q / k / v,
+// attention-output and MLP buffers hold each branch's joint sequence [text; image].
 static const float* br_mod(const bag_ctx* ctx, int br) { return br ? ctx->mod_all_u : ctx->mod_all; }
 static const void* br_txt(const bag_ctx* ctx, int br) { return br ? ctx->txt_stage_u : ctx->txt_stage; }
 static int n_branches(const bag_ctx* ctx) { return ctx->arch.cfg ? 2 : 1; }
 
-// One block of the stack on the stream h (joint [N, d] with text rows first, or the
-// Wan image stream [ni, d]) with branch br's modulation and (Wan) context.
-static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int br = 0) {
+// Branch-map fields of an epilogue whose problem holds nb branches of `rows` rows each.
+static void epi_branches(const bag_ctx* ctx, Epi& e, int nb, int rows, long qk_rows, long vpad) {
+  if (nb < 2) return;
+  e.br_rows = rows;
+  e.br_qk = qk_rows;
+  e.br_vt = (long)ctx->H * ctx->dh * vpad;  // used only for transposed V (v_mode 1)
+}
+
+// One block of the stack on the stream h for nb branches (1: the joint [N, d] sequence
+// with text rows first, or the Wan image stream [ni, d]; 2: both guidance branches in
+// the order above), with each branch's modulation and (Wan) context.
+static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int nb = 1) {
   bag_ctx* ctx = q.ctx;
   const Block& blk = ctx->blocks[b];
   const long d = ctx->d, F = ctx->F, ldc = d + F;
   const int ni = ctx->ni, nx = ctx->nx, N = ctx->N;
-  const float* mod = br_mod(ctx, br) + blk.mod_off;
+  const float* mod = ctx->mod_all + blk.mod_off;                     // branch 0
+  const float* modu = br_mod(ctx, nb > 1 ? 1 : 0) + blk.mod_off;      // branch 1 (or 0)
   const long ms = ctx->mod_stride;
+  // element offset of branch 1's V: transposed per head for the tensor-core attention
+  // (H x dh x vpad), else row-major like k (rows x d)
+  auto v_br = [&](long rows, long vpad) { return ctx->act_bf16 ? (long)ctx->H * ctx->dh * vpad : rows * d; };
+  const long vt_br = v_br(N, ctx->vpad);
   // QK-norm scales of a stream (pre = "", "img_" or "txt_"), when the block has them
   auto qk_norm = [&](Epi& e, const std::string& pre) {
     auto it = blk.w.find(pre + "q_norm");
@@ -892,43 +945,91 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int b
     e.qn_q = (const float*)it->second.p;
     e.qn_k = (const float*)blk.w.at(pre + "k_norm").p;
   };
+  // LayerNorm + modulation of the joint stream (nb * N rows) with the text rows of each
+  // branch under (sh_t, sc_t) + offset and the image rows under (sh_i, sc_i) + offset
+  auto ln_joint = [&](const float* mt_c, const float* mt_u, const float* mi_c, const float* mi_u,
+                      long off) {
+    if (nb == 1) {
+      enq_ln(q, h, d, ctx->xn, d, N, nx, mt_c + off, mt_c + off + d, mi_c + off, mi_c + off + d, st, fw);
+      return;
+    }
+    enq_ln4(q, h, d, ctx->xn, d, 2 * N, nx, 2 * nx, 2 * nx + ni, mt_c + off, mt_u + off, mi_c + off,
+            mi_u + off, st, fw);
+  };
+  // attention of every branch: q / k / v of branch br at row br * N (transposed V at
+  // br * vt_br); the output rows go back in stream order (text rows of branch br at
+  // br * nx, its image rows at nb * nx + br * ni)
+  auto attn_joint = [&]() {
+    for (int br = 0; br < nb; ++br) {
+      void* o = off_act(ctx, ctx->cat, (long)br * nx * ldc);
+      void* o2 = off_act(ctx, ctx->cat, ((long)nb * nx + (long)br * ni - nx) * ldc);
+      enq_attn(q, off_act(ctx, ctx->q, (long)br * N * d), off_act(ctx, ctx->k, (long)br * N * d),
+               off_act(ctx, ctx->vt, br * vt_br), ctx->vpad, o, ldc, N, N, st, fw,
+               nb > 1 ? o2 : nullptr, nx);
+    }
+  };
   if (blk.type == BT_SINGLE) {
-    enq_ln(q, h, d, ctx->xn, d, N, 0, mod, mod + d, mod, mod + d, st, fw);
+    ln_joint(mod, modu, mod, modu, 0);
     Epi e = base_epi(ctx, st, fw);
     enq_qkv_epi(ctx, e, 0, true);
     qk_norm(e, "");
-    enq_gemm(q, ctx->xn, d, blk.w.at("lin1_w"), d, N, (int)(3 * d + F), (int)d,
-             (e.bias = (const float*)blk.w.at("lin1_b").p, e));
-    enq_attn(q, ctx->q, ctx->k, ctx->vt, ctx->vpad, ctx->cat, ldc, N, N, st, fw);
+    e.bias = (const float*)blk.w.at("lin1_b").p;
     Epi r = base_epi(ctx, st, fw);
     r.kind = EPI_GATED_RES;
     r.bias = (const float*)blk.w.at("lin2_b").p;
     r.resid = h;
     r.ldr = d;
     r.gate = mod + 2 * d;
+    r.gate_u = modu + 2 * d;
     r.gate_step = ms;
-    enq_gemm(q, ctx->cat, ldc, blk.w.at("lin2_w"), ldc, N, (int)d, (int)(d + F), r);
+    if (nb == 1) {
+      enq_gemm(q, ctx->xn, d, blk.w.at("lin1_w"), d, N, (int)(3 * d + F), (int)d, e);
+      attn_joint();
+      enq_gemm(q, ctx->cat, ldc, blk.w.at("lin2_w"), ldc, N, (int)d, (int)(d + F), r);
+      return;
+    }
+    // both branches: the text rows and the image rows as two problems of one launch
+    // (the same weight), each covering the two branches
+    Epi ei = e;
+    ei.row_off = nx;
+    ei.mlp = off_act(ctx, ctx->cat, 2L * nx * ldc + d);
+    epi_branches(ctx, ei, nb, ni, N, ctx->vpad);
+    epi_branches(ctx, e, nb, nx, N, ctx->vpad);
+    enq_gemm2(q, off_act(ctx, ctx->xn, 2L * nx * d), d, blk.w.at("lin1_w"), d, 2 * ni, ei,
+              ctx->xn, d, blk.w.at("lin1_w"), d, 2 * nx, e, (int)(3 * d + F), (int)d);
+    attn_joint();
+    Epi ri = r;
+    ri.resid = h + 2L * nx * d;
+    ri.br_rows = ni;
+    r.br_rows = nx;
+    enq_gemm2(q, off_act(ctx, ctx->cat, 2L * nx * ldc), ldc, blk.w.at("lin2_w"), ldc, 2 * ni, ri,
+              ctx->cat, ldc, blk.w.at("lin2_w"), ldc, 2 * nx, r, (int)d, (int)(d + F));
     return;
   }
   if (blk.type == BT_DOUBLE) {
-    const float* mi = mod;           // image stream modulation (6d)
-    const float* mt = mod + 6 * d;   // text stream modulation (6d)
-    float* h_img = h + (long)nx * d;
+    const float* mi = mod;              // image stream modulation (6d), branch 0
+    const float* mt = mod + 6 * d;      // text stream modulation (6d), branch 0
+    const float* miu = modu;            // branch 1
+    const float* mtu = modu + 6 * d;
+    const long ti = (long)nb * nx;      // first image row of the stream
+    float* h_img = h + ti * d;
     // attention half
-    enq_ln(q, h, d, ctx->xn, d, N, nx, mt, mt + d, mi, mi + d, st, fw);
+    ln_joint(mt, mtu, mi, miu, 0);
     {
       Epi e = base_epi(ctx, st, fw);
       enq_qkv_epi(ctx, e, nx, true);
       e.bias = (const float*)blk.w.at("img_qkv_b").p;
       qk_norm(e, "img_");
+      epi_branches(ctx, e, nb, ni, N, ctx->vpad);
       Epi e2 = base_epi(ctx, st, fw);
       enq_qkv_epi(ctx, e2, 0, true);
       e2.bias = (const float*)blk.w.at("txt_qkv_b").p;
       qk_norm(e2, "txt_");
-      enq_gemm2(q, off_act(ctx, ctx->xn, (long)nx * d), d, blk.w.at("img_qkv_w"), d, ni, e,
-                ctx->xn, d, blk.w.at("txt_qkv_w"), d, nx, e2, (int)(3 * d), (int)d);
+      epi_branches(ctx, e2, nb, nx, N, ctx->vpad);
+      enq_gemm2(q, off_act(ctx, ctx->xn, ti * d), d, blk.w.at("img_qkv_w"), d, nb * ni, e,
+                ctx->xn, d, blk.w.at("txt_qkv_w"), d, nb * nx, e2, (int)(3 * d), (int)d);
     }
-    enq_attn(q, ctx->q, ctx->k, ctx->vt, ctx->vpad, ctx->cat, ldc, N, N, st, fw);
+    attn_joint();
     {
       Epi r = base_epi(ctx, st, fw);
       r.kind = EPI_GATED_RES;
@@ -936,53 +1037,68 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int b
       r.resid = h_img;
       r.ldr = d;
       r.gate = mi + 2 * d;
+      r.gate_u = miu + 2 * d;
       r.gate_step = ms;
+      if (nb > 1) r.br_rows = ni;
       Epi r2 = r;
       r2.bias = (const float*)blk.w.at("txt_proj_b").p;
       r2.resid = h;
       r2.gate = mt + 2 * d;
-      enq_gemm2(q, off_act(ctx, ctx->cat, (long)nx * ldc), ldc, blk.w.at("img_proj_w"), d, ni, r,
-                ctx->cat, ldc, blk.w.at("txt_proj_w"), d, nx, r2, (int)d, (int)d);
+      r2.gate_u = mtu + 2 * d;
+      if (nb > 1) r2.br_rows = nx;
+      enq_gemm2(q, off_act(ctx, ctx->cat, ti * ldc), ldc, blk.w.at("img_proj_w"), d, nb * ni, r,
+                ctx->cat, ldc, blk.w.at("txt_proj_w"), d, nb * nx, r2, (int)d, (int)d);
     }
     // MLP half
-    enq_ln(q, h, d, ctx->xn, d, N, nx, mt + 3 * d, mt + 4 * d, mi + 3 * d, mi + 4 * d, st, fw);
+    ln_joint(mt, mtu, mi, miu, 3 * d);
     {
       Epi u = base_epi(ctx, st, fw);
       u.kind = EPI_GELU;
       u.out_bf16 = ctx->act_bf16;
       u.ldo = ldc;
       u.bias = (const float*)blk.w.at("img_up_b").p;
-      u.out = off_act(ctx, ctx->cat, (long)nx * ldc + d);
+      u.out = off_act(ctx, ctx->cat, ti * ldc + d);
       Epi u2 = u;
       u2.bias = (const float*)blk.w.at("txt_up_b").p;
       u2.out = off_act(ctx, ctx->cat, d);
-      enq_gemm2(q, off_act(ctx, ctx->xn, (long)nx * d), d, blk.w.at("img_up_w"), d, ni, u,
-                ctx->xn, d, blk.w.at("txt_up_w"), d, nx, u2, (int)F, (int)d);
+      enq_gemm2(q, off_act(ctx, ctx->xn, ti * d), d, blk.w.at("img_up_w"), d, nb * ni, u,
+                ctx->xn, d, blk.w.at("txt_up_w"), d, nb * nx, u2, (int)F, (int)d);
       Epi r = base_epi(ctx, st, fw);
       r.kind = EPI_GATED_RES;
       r.bias = (const float*)blk.w.at("img_down_b").p;
       r.resid = h_img;
       r.ldr = d;
       r.gate = mi + 5 * d;
+      r.gate_u = miu + 5 * d;
       r.gate_step = ms;
+      if (nb > 1) r.br_rows = ni;
       Epi r2 = r;
       r2.bias = (const float*)blk.w.at("txt_down_b").p;
       r2.resid = h;
       r2.gate = mt + 5 * d;
-      enq_gemm2(q, off_act(ctx, ctx->cat, (long)nx * ldc + d), ldc, blk.w.at("img_down_w"), F, ni, r,
-                off_act(ctx, ctx->cat, d), ldc, blk.w.at("txt_down_w"), F, nx, r2, (int)d, (int)F);
+      r2.gate_u = mtu + 5 * d;
+      if (nb > 1) r2.br_rows = nx;
+      enq_gemm2(q, off_act(ctx, ctx->cat, ti * ldc + d), ldc, blk.w.at("img_down_w"), F, nb * ni, r,
+                off_act(ctx, ctx->cat, d), ldc, blk.w.at("txt_down_w"), F, nb * nx, r2, (int)d, (int)F);
     }
     return;
   }
-  // Wan block: self-attention, cross-attention, FFN
-  enq_ln(q, h, d, ctx->xn, d, ni, 0, mod, mod + d, mod, mod + d, st, fw);
+  // Wan block: self-attention, cross-attention, FFN; under guidance the stream holds
+  // [image_c; image_u] and the staged contexts [context_c; context_u]
+  const int R = nb * ni;
+  const long vtw_br = v_br(ni, ctx->vpad), vtc_br = v_br(nx, ctx->vpad_c);
+  enq_ln(q, h, d, ctx->xn, d, R, ni, mod, mod + d, modu, modu + d, st, fw);
   {
     Epi e = base_epi(ctx, st, fw);
     enq_qkv_epi(ctx, e, 0, true);
     e.bias = (const float*)blk.w.at("sa_qkv_b").p;
-    enq_gemm(q, ctx->xn, d, blk.w.at("sa_qkv_w"), d, ni, (int)(3 * d), (int)d, e);
+    epi_branches(ctx, e, nb, ni, ni, ctx->vpad);
+    enq_gemm(q, ctx->xn, d, blk.w.at("sa_qkv_w"), d, R, (int)(3 * d), (int)d, e);
   }
-  enq_attn(q, ctx->q, ctx->k, ctx->vt, ctx->vpad, ctx->cat, ldc, ni, ni, st, fw);
+  for (int br = 0; br < nb; ++br)
+    enq_attn(q, off_act(ctx, ctx->q, (long)br * ni * d), off_act(ctx, ctx->k, (long)br * ni * d),
+             off_act(ctx, ctx->vt, br * vtw_br), ctx->vpad, off_act(ctx, ctx->cat, (long)br * ni * ldc),
+             ldc, ni, ni, st, fw);
   {
     Epi r = base_epi(ctx, st, fw);
     r.kind = EPI_GATED_RES;
@@ -990,10 +1106,12 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int b
     r.resid = h;
     r.ldr = d;
     r.gate = mod + 2 * d;
+    r.gate_u = modu + 2 * d;
     r.gate_step = ms;
-    enq_gemm(q, ctx->cat, ldc, blk.w.at("sa_o_w"), d, ni, (int)d, (int)d, r);
+    if (nb > 1) r.br_rows = ni;
+    enq_gemm(q, ctx->cat, ldc, blk.w.at("sa_o_w"), d, R, (int)d, (int)d, r);
   }
-  enq_ln(q, h, d, ctx->xn, d, ni, 0, nullptr, nullptr, nullptr, nullptr, st, fw);
+  enq_ln(q, h, d, ctx->xn, d, R, 0, nullptr, nullptr, nullptr, nullptr, st, fw);
   {
     Epi e = base_epi(ctx, st, fw);
     e.kind = EPI_STORE;
@@ -1001,7 +1119,7 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int b
     e.ldo = d;
     e.out_bf16 = ctx->act_bf16 ? kStoreF16 : kStoreF32;  // an attention operand
     e.bias = (const float*)blk.w.at("ca_q_b").p;
-    enq_gemm(q, ctx->xn, d, blk.w.at("ca_q_w"), d, ni, (int)d, (int)d, e);
+    enq_gemm(q, ctx->xn, d, blk.w.at("ca_q_w"), d, R, (int)d, (int)d, e);
     Epi kv = base_epi(ctx, st, fw);
     kv.kind = EPI_QKV;
     kv.q = nullptr;
@@ -1016,18 +1134,22 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int b
     kv.col_base = (int)d;
     kv.rope = nullptr;
     kv.bias = (const float*)blk.w.at("ca_kv_b").p;
-    enq_gemm(q, br_txt(ctx, br), d, blk.w.at("ca_kv_w"), d, nx, (int)(2 * d), (int)d, kv);
+    epi_branches(ctx, kv, nb, nx, nx, ctx->vpad_c);
+    enq_gemm(q, ctx->txt_stage, d, blk.w.at("ca_kv_w"), d, nb * nx, (int)(2 * d), (int)d, kv);
   }
-  enq_attn(q, ctx->qc, ctx->kc, ctx->vtc, ctx->vpad_c, ctx->cat, ldc, ni, nx, st, fw);
+  for (int br = 0; br < nb; ++br)
+    enq_attn(q, off_act(ctx, ctx->qc, (long)br * ni * d), off_act(ctx, ctx->kc, (long)br * nx * d),
+             off_act(ctx, ctx->vtc, br * vtc_br), ctx->vpad_c, off_act(ctx, ctx->cat, (long)br * ni * ldc),
+             ldc, ni, nx, st, fw);
   {
     Epi r = base_epi(ctx, st, fw);
     r.kind = EPI_RES_ADD;
     r.bias = (const float*)blk.w.at("ca_o_b").p;
     r.resid = h;
     r.ldr = d;
-    enq_gemm(q, ctx->cat, ldc, blk.w.at("ca_o_w"), d, ni, (int)d, (int)d, r);
+    enq_gemm(q, ctx->cat, ldc, blk.w.at("ca_o_w"), d, R, (int)d, (int)d, r);
   }
-  enq_ln(q, h, d, ctx->xn, d, ni, 0, mod + 3 * d, mod + 4 * d, mod + 3 * d, mod + 4 * d, st, fw);
+  enq_ln(q, h, d, ctx->xn, d, R, ni, mod + 3 * d, mod + 4 * d, modu + 3 * d, modu + 4 * d, st, fw);
   {
     Epi u = base_epi(ctx, st, fw);
     u.kind = EPI_GELU;
@@ -1035,21 +1157,24 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int b
     u.ldo = ldc;
     u.bias = (const float*)blk.w.at("ffn_up_b").p;
     u.out = off_act(ctx, ctx->cat, d);
-    enq_gemm(q, ctx->xn, d, blk.w.at("ffn_up_w"), d, ni, (int)F, (int)d, u);
+    enq_gemm(q, ctx->xn, d, blk.w.at("ffn_up_w"), d, R, (int)F, (int)d, u);
     Epi r = base_epi(ctx, st, fw);
     r.kind = EPI_GATED_RES;
     r.bias = (const float*)blk.w.at("ffn_down_b").p;
     r.resid = h;
     r.ldr = d;
     r.gate = mod + 5 * d;
+    r.gate_u = modu + 5 * d;
     r.gate_step = ms;
-    enq_gemm(q, off_act(ctx, ctx->cat, d), ldc, blk.w.at("ffn_down_w"), F, ni, (int)d, (int)F, r);
+    if (nb > 1) r.br_rows = ni;
+    enq_gemm(q, off_act(ctx, ctx->cat, d), ldc, blk.w.at("ffn_down_w"), F, R, (int)d, (int)F, r);
   }
 }
 
+// Image rows of branch br in the stream (text rows of branch br start at br * nx).
 static float* img_stream(bag_ctx* ctx, int br = 0) {
-  float* h = br_stream(ctx, br);
-  return ctx->arch.kind == BAG_KIND_WAN ? h : h + (long)ctx->nx * ctx->d;
+  if (ctx->arch.kind == BAG_KIND_WAN) return ctx->hj + (long)br * ctx->ni * ctx->d;
+  return ctx->hj + ((long)n_branches(ctx) * ctx->nx + (long)br * ctx->ni) * ctx->d;
 }
 
 static void enq_prefix(Enq& q, int use_cond, unsigned long long handle) {
@@ -1114,15 +1239,19 @@ static void enq_prefix(Enq& q, int use_cond, unsigned long long handle) {
 static void enq_full(Enq& q, int fw) {
   bag_ctx* ctx = q.ctx;
   const long d = ctx->d;
-  for (int br = 0; br < n_branches(ctx); ++br) {
-    float* h = br_stream(ctx, br);
+  const int nb = n_branches(ctx);
+  for (int br = 0; br < nb; ++br) {
     if (ctx->arch.kind != BAG_KIND_WAN)
-      q.chk(copy_rows_f32(ctx->st, fw, h, d, br_txt(ctx, br), d, ctx->act_bf16, ctx->nx, (int)d, q.s));
+      q.chk(copy_rows_f32(ctx->st, fw, ctx->hj + (long)br * ctx->nx * d, d, br_txt(ctx, br), d, ctx->act_bf16,
+                          ctx->nx, (int)d, q.s));
     if (br) {  // the patch-embed epilogue filled only the conditional stream's image rows
       q.pre(BAG_PROF_CACHE, 0.0, (double)ctx->ni * d * 8.0);
       q.chk(copy_rows_f32(ctx->st, fw, img_stream(ctx, br), d, ctx->h_in, d, 0, ctx->ni, (int)d, q.s));
     }
-    for (int b = 0; b < ctx->nblk; ++b) enq_block(q, b, h, ctx->st, fw, br);
+  }
+  // the stack once for all branches (every projection takes both branches' rows)
+  for (int b = 0; b < ctx->nblk; ++b) enq_block(q, b, ctx->hj, ctx->st, fw, nb);
+  for (int br = 0; br < nb; ++br) {
     q.pre(BAG_PROF_CACHE, 0.0, (double)ctx->ni * d * 12.0);
     q.chk(cache_refresh(ctx->st, img_stream(ctx, br), ctx->h_in, br ? ctx->R_u : ctx->R,
                         (long)ctx->ni * d, fw, q.s));

@@ -128,9 +128,21 @@ __global__ void __launch_bounds__(LN_THREADS, VPT <= 6 ? 8 : (VPT <= 10 ? 5 : 4)
   }
   // the previous step was fully computed: its observable (ref2) is the new reference
   const bool refresh = a.sig_on && a.sig_ref_w && a.st && a.st->t > 0 && a.st->t_last == a.st->t - 1;
-  const bool first = row < a.split;
-  const float* sh = first ? a.shift_a : a.shift_b;
-  const float* sc = first ? a.scale_a : a.scale_b;
+  const float* sh;
+  const float* sc;
+  if (row < a.split) {
+    sh = a.shift_a;
+    sc = a.scale_a;
+  } else if (a.split2 <= 0 || row < a.split2) {
+    sh = a.shift_b;
+    sc = a.scale_b;
+  } else if (row < a.split3) {
+    sh = a.shift_c;
+    sc = a.scale_c;
+  } else {
+    sh = a.shift_d;
+    sc = a.scale_d;
+  }
   if (sh) sh += (long)t * a.mod_step;
   if (sc) sc += (long)t * a.mod_step;
   float sig_num = 0.f, sig_den = 0.f, sig_num2 = 0.f, sig_den2 = 0.f;

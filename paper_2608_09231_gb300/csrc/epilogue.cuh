@@ -167,27 +167,29 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float r
         store_vals<NV>(e.mlp, (long)row * e.ldm + (lc - 3 * e.d), v, e.act_bf16);
         break;
       }
-      const int jr = row + e.row_off;  // joint-sequence row
+      const bool br1 = e.br_rows > 0 && row >= e.br_rows;       // unconditional branch
+      const int jr = row - (br1 ? e.br_rows : 0) + e.row_off;  // joint-sequence row
+      const long qr = jr + (br1 ? e.br_qk : 0);                // q / k / v buffer row
       const int cc = lc - region * e.d;
       if (region < 2) epi_qk_transform<NV>(e, jr, cc, region, v, rs);
       if (region == 0) {
-        store_vals<NV>(e.q, (long)jr * e.ldqk + cc, v, e.qkv_type);
+        store_vals<NV>(e.q, qr * e.ldqk + cc, v, e.qkv_type);
       } else if (region == 1) {
-        store_vals<NV>(e.k, (long)jr * e.ldqk + cc, v, e.qkv_type);
+        store_vals<NV>(e.k, qr * e.ldqk + cc, v, e.qkv_type);
       } else if (e.v_mode == 0) {
-        store_vals<NV>(e.v, (long)jr * e.ldqk + cc, v, e.qkv_type);
+        store_vals<NV>(e.v, qr * e.ldqk + cc, v, e.qkv_type);
       } else {
         // transposed per head: vt[(head * dh + e) * vpad + token]
         if (e.qkv_type == kStoreF16) {
-          __half* vt = reinterpret_cast<__half*>(e.v);
+          __half* vt = reinterpret_cast<__half*>(e.v) + (br1 ? e.br_vt : 0);
 #pragma unroll
           for (int j = 0; j < NV; ++j) vt[(long)(cc + j) * e.vpad + jr] = __float2half_rn(v[j]);
         } else if (e.qkv_type == kStoreBF16) {
-          __nv_bfloat16* vt = reinterpret_cast<__nv_bfloat16*>(e.v);
+          __nv_bfloat16* vt = reinterpret_cast<__nv_bfloat16*>(e.v) + (br1 ? e.br_vt : 0);
 #pragma unroll
           for (int j = 0; j < NV; ++j) vt[(long)(cc + j) * e.vpad + jr] = __float2bfloat16_rn(v[j]);
         } else {
-          float* vt = reinterpret_cast<float*>(e.v);
+          float* vt = reinterpret_cast<float*>(e.v) + (br1 ? e.br_vt : 0);
 #pragma unroll
           for (int j = 0; j < NV; ++j) vt[(long)(cc + j) * e.vpad + jr] = v[j];
         }
@@ -195,7 +197,7 @@ BAG_DEV void epi_apply(const Epi& e, int t, int row, int col0, float* v, float r
       break;
     }
     case EPI_GATED_RES: {
-      const float* g = e.gate + (long)t * e.gate_step + col0;
+      const float* g = (e.br_rows > 0 && row >= e.br_rows ? e.gate_u : e.gate) + (long)t * e.gate_step + col0;
       float* r = e.resid + (long)row * e.ldr + col0;
       if (NV % 4 == 0 && ((reinterpret_cast<uintptr_t>(g) | reinterpret_cast<uintptr_t>(r)) & 15) == 0) {
 #pragma unroll

@@ -157,6 +157,34 @@ static int tile_group_rows(int M, int BM, int K, int a_split) {
 constexpr int kVtScratchFloats = 32 * 33;
 constexpr int kVtScratchBytes = 4 * kVtScratchFloats * 4;  // four epilogue warps
 
+BAG_DEV uint16_t to16(float x, bool f16) {
+  return f16 ? __half_as_ushort(__float2half_rn(x)) : __bfloat16_as_ushort(__float2bfloat16_rn(x));
+}
+BAG_DEV uint32_t pack16x2(float a, float b, bool f16) { return f16 ? pack_f16x2(a, b) : pack_bf16x2(a, b); }
+
+// 32 consecutive 16-bit tokens of one V^T row starting at dst, whose address is MIS
+// elements past a 16-byte boundary: the elements before the first boundary and after
+// the last one singly, everything between as 16-byte stores.
+template <int MIS>
+BAG_DEV void store_vt_run(uint16_t* dst, const float* tc, bool f16) {
+  constexpr int H = (8 - MIS) & 7;   // elements before the first 16-byte boundary
+  constexpr int NCH = (32 - H) / 8;  // whole 16-byte chunks
+#pragma unroll
+  for (int k = 0; k < H; ++k) dst[k] = to16(tc[k], f16);
+#pragma unroll
+  for (int c = 0; c < NCH; ++c) {
+    const int k = H + 8 * c;
+    uint4 w;
+    w.x = pack16x2(tc[k], tc[k + 1], f16);
+    w.y = pack16x2(tc[k + 2], tc[k + 3], f16);
+    w.z = pack16x2(tc[k + 4], tc[k + 5], f16);
+    w.w = pack16x2(tc[k + 6], tc[k + 7], f16);
+    *reinterpret_cast<uint4*>(dst + k) = w;
+  }
+#pragma unroll
+  for (int k = H + 8 * NCH; k < 32; ++k) dst[k] = to16(tc[k], f16);
+}
+
 // V columns of a QKV projection with 16-bit (bf16 or fp16) storage, stored transposed per head
 // (vt[(head * dh + e) * vpad + token]): the warp's 32 rows x 32 columns pass through
 // shared memory, so each lane writes one column's 32 consecutive tokens as four 16-byte
@@ -176,24 +204,38 @@ BAG_DEV void store_vt_warp(const Epi& e, int row, int col, float* v, float* sbuf
   for (int k = 0; k < 32; ++k) tc[k] = sbuf[lane * 33 + k];
   __syncwarp();
   const int row0 = row - lane;
-  const int jr0 = row0 + e.row_off;
+  // guidance branches (br_rows > 0): the warp's 32 rows take the fast path only when
+  // they all belong to one branch
+  const bool br1 = e.br_rows > 0 && row0 >= e.br_rows;
+  const bool one_branch = e.br_rows == 0 || br1 || row0 + 31 < e.br_rows;
+  const int jr0 = row0 - (br1 ? e.br_rows : 0) + e.row_off;
   const int cc = col + e.col_base - 2 * e.d + lane;  // this lane's column within V
   const bool f16 = e.qkv_type == kStoreF16;
-  uint16_t* dst = reinterpret_cast<uint16_t*>(e.v) + (long)cc * e.vpad + jr0;
-  if (row0 + 31 < e.M && (jr0 & 7) == 0) {
-    uint4 w[4];
-    uint32_t* wp = reinterpret_cast<uint32_t*>(w);
-#pragma unroll
-    for (int k = 0; k < 16; ++k)
-      wp[k] = f16 ? pack_f16x2(tc[2 * k], tc[2 * k + 1]) : pack_bf16x2(tc[2 * k], tc[2 * k + 1]);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) reinterpret_cast<uint4*>(dst)[k] = w[k];
+  uint16_t* vbase = reinterpret_cast<uint16_t*>(e.v);
+  uint16_t* dst = vbase + (br1 ? e.br_vt : 0) + (long)cc * e.vpad + jr0;
+  if (row0 + 31 < e.M && one_branch) {
+    // dst is 16-byte aligned exactly when jr0 is a multiple of 8 (vpad and the branch
+    // offset are multiples of 8 elements)
+    switch (jr0 & 7) {
+      case 0: store_vt_run<0>(dst, tc, f16); break;
+      case 1: store_vt_run<1>(dst, tc, f16); break;
+      case 2: store_vt_run<2>(dst, tc, f16); break;
+      case 3: store_vt_run<3>(dst, tc, f16); break;
+      case 4: store_vt_run<4>(dst, tc, f16); break;
+      case 5: store_vt_run<5>(dst, tc, f16); break;
+      case 6: store_vt_run<6>(dst, tc, f16); break;
+      default: store_vt_run<7>(dst, tc, f16); break;
+    }
   } else {
 #pragma unroll
-    for (int k = 0; k < 32; ++k)
-      if (row0 + k < e.M)
-        dst[k] = f16 ? __half_as_ushort(__float2half_rn(tc[k]))
-                     : __bfloat16_as_ushort(__float2bfloat16_rn(tc[k]));
+    for (int k = 0; k < 32; ++k) {
+      const int rk = row0 + k;
+      if (rk < e.M) {
+        const bool b1 = e.br_rows > 0 && rk >= e.br_rows;
+        const long at = (b1 ? e.br_vt : 0) + (long)cc * e.vpad + rk - (b1 ? e.br_rows : 0) + e.row_off;
+        vbase[at] = to16(tc[k], f16);
+      }
+    }
   }
 }
 

@@ -93,6 +93,7 @@ struct Epi {
   float* resid = nullptr;
   long ldr = 0;
   const float* gate = nullptr;    // gate for step t = gate + t * gate_step
+  const float* gate_u = nullptr;  // unconditional branch's gate (rows >= br_rows)
   long gate_step = 0;
   // attention operands
   void* q = nullptr;
@@ -103,6 +104,12 @@ struct Epi {
   int d = 0, dh = 0;
   long vpad = 0;
   int row_off = 0;         // joint-sequence row of this GEMM's row 0
+  // Two guidance branches in one problem: rows [0, br_rows) are the conditional branch,
+  // rows [br_rows, 2 br_rows) the unconditional one (br_rows = 0: a single branch).
+  // EPI_QKV writes branch 1's q / k rows br_qk rows further and its transposed V br_vt
+  // elements further; EPI_GATED_RES takes branch 1's gate from gate_u.
+  int br_rows = 0;
+  long br_qk = 0, br_vt = 0;
   int col_base = 0;        // logical column of this GEMM's column 0 (q=0, k=d, v=2d, mlp=3d)
   const float2* rope = nullptr;  // [joint rows][dh/2] (cos, sin); null = no rotation
   int act_bf16 = 1;        // mlp storage type (1 bf16, 0 fp32)
@@ -157,6 +164,7 @@ struct AttnArgs {
   const void* k;  long ldk;      // [Nk rows][ldk]
   const void* v;  int v_mode; long ldv; long vpad;  // mode 0 like k; mode 1 [H][dh][vpad]
   void* o;        long ldo;      // output [Nq][ldo], head h at column h*dh
+  void* o2 = nullptr; int o_split = 0;  // rows >= o_split go to o2 (+ row * ldo) instead
   int nq, nk, heads, dh;
   int bf16;                      // 16-bit operands and output (else fp32)
   int f16 = 0;                   // with bf16: q, k, v are fp16 (output stays bf16)
@@ -174,6 +182,11 @@ struct LnArgs {
   int rows, cols, split;
   const float* shift_a; const float* scale_a;
   const float* shift_b; const float* scale_b;
+  // up to four row segments: [0, split) a, [split, split2) b, [split2, split3) c,
+  // [split3, rows) d (split2 = split3 = 0: two segments)
+  int split2 = 0, split3 = 0;
+  const float* shift_c = nullptr; const float* scale_c = nullptr;
+  const float* shift_d = nullptr; const float* scale_d = nullptr;
   long mod_step;
   // fused trajectory signal: per-row partial sums of |y - ref|, |ref|, |y - ref2|,
   // |ref2| (4 floats per row); ref2 may alias y (it is read before y is stored).
