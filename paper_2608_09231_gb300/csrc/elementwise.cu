@@ -37,8 +37,23 @@ BAG_DEV float block_sum(float v, float* red) {
   return s;
 }
 
+// Block-wide sum through a shared array that this CTA uses for nothing else: one barrier
+// (no barrier is needed before the writes, since no earlier reduction reads the array).
+BAG_DEV float block_sum_fresh(float v, float* red) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float s = 0.f;
+#pragma unroll
+  for (int w = 0; w < LN_THREADS / 32; ++w) s += red[w];
+  return s;
+}
+
 // Four block-wide sums at once (one pair of barriers instead of four).
-BAG_DEV float4 block_sum4(float4 v, float4* red) {
+// fresh: red is used by no earlier reduction of the CTA, so no barrier precedes the writes.
+BAG_DEV float4 block_sum4(float4 v, float4* red, bool fresh_red = false) {
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
     v.x += __shfl_xor_sync(0xffffffffu, v.x, off);
@@ -47,7 +62,7 @@ BAG_DEV float4 block_sum4(float4 v, float4* red) {
     v.w += __shfl_xor_sync(0xffffffffu, v.w, off);
   }
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  __syncthreads();
+  if (!fresh_red) __syncthreads();
   if (lane == 0) red[warp] = v;
   __syncthreads();
   float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -96,7 +111,8 @@ template <int VPT>
 __global__ void __launch_bounds__(LN_THREADS, VPT <= 6 ? 8 : (VPT <= 10 ? 5 : 4)) ln_mod_kernel(const LnArgs a) {
   grid_dep_sync();
   if (epi_skip(a.st, a.flag_want)) return;
-  __shared__ float red[LN_THREADS / 32];
+  // one shared array per reduction of the row, so that each takes a single barrier
+  __shared__ float red_mean[LN_THREADS / 32], red_var[LN_THREADS / 32];
   const int row = blockIdx.x;
   if (row >= a.rows) return;
   const int t = a.st ? a.st->t : 0;
@@ -114,7 +130,7 @@ __global__ void __launch_bounds__(LN_THREADS, VPT <= 6 ? 8 : (VPT <= 10 ? 5 : 4)
   }
   float mean = 0.f, rstd = 1.f;  // identity: y = x
   if (!a.identity) {
-    mean = block_sum(s, red) / (float)a.cols;
+    mean = block_sum_fresh(s, red_mean) / (float)a.cols;
     float q = 0.f;
 #pragma unroll
     for (int i = 0; i < VPT; ++i) {
@@ -124,7 +140,7 @@ __global__ void __launch_bounds__(LN_THREADS, VPT <= 6 ? 8 : (VPT <= 10 ? 5 : 4)
         q += (dx * dx + dy * dy) + (dz * dz + dw * dw);
       }
     }
-    rstd = rsqrtf(block_sum(q, red) / (float)a.cols + 1e-6f);
+    rstd = rsqrtf(block_sum_fresh(q, red_var) / (float)a.cols + 1e-6f);
   }
   // the previous step was fully computed: its observable (ref2) is the new reference
   const bool refresh = a.sig_on && a.sig_ref_w && a.st && a.st->t > 0 && a.st->t_last == a.st->t - 1;
@@ -201,7 +217,7 @@ __global__ void __launch_bounds__(LN_THREADS, VPT <= 6 ? 8 : (VPT <= 10 ? 5 : 4)
   }
   if (a.sig_on) {
     __shared__ float4 red4[LN_THREADS / 32];
-    const float4 t4 = block_sum4(make_float4(sig_num, sig_den, sig_num2, sig_den2), red4);
+    const float4 t4 = block_sum4(make_float4(sig_num, sig_den, sig_num2, sig_den2), red4, true);
     if (threadIdx.x == 0) reinterpret_cast<float4*>(a.sig_partial)[row] = t4;
   }
 }

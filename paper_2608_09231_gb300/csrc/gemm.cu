@@ -162,27 +162,28 @@ BAG_DEV uint16_t to16(float x, bool f16) {
 }
 BAG_DEV uint32_t pack16x2(float a, float b, bool f16) { return f16 ? pack_f16x2(a, b) : pack_bf16x2(a, b); }
 
-// 32 consecutive 16-bit tokens of one V^T row starting at dst, whose address is MIS
-// elements past a 16-byte boundary: the elements before the first boundary and after
-// the last one singly, everything between as 16-byte stores.
-template <int MIS>
+// 32 consecutive 16-bit tokens of one V^T row starting at dst: 16-byte stores when dst is
+// 16-byte aligned, else 4-byte stores (with a single leading element when dst is odd).
 BAG_DEV void store_vt_run(uint16_t* dst, const float* tc, bool f16) {
-  constexpr int H = (8 - MIS) & 7;   // elements before the first 16-byte boundary
-  constexpr int NCH = (32 - H) / 8;  // whole 16-byte chunks
+  if ((reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
 #pragma unroll
-  for (int k = 0; k < H; ++k) dst[k] = to16(tc[k], f16);
+    for (int k = 0; k < 32; k += 8) {
+      uint4 w;
+      w.x = pack16x2(tc[k], tc[k + 1], f16);
+      w.y = pack16x2(tc[k + 2], tc[k + 3], f16);
+      w.z = pack16x2(tc[k + 4], tc[k + 5], f16);
+      w.w = pack16x2(tc[k + 6], tc[k + 7], f16);
+      *reinterpret_cast<uint4*>(dst + k) = w;
+    }
+  } else if ((reinterpret_cast<uintptr_t>(dst) & 3) == 0) {
 #pragma unroll
-  for (int c = 0; c < NCH; ++c) {
-    const int k = H + 8 * c;
-    uint4 w;
-    w.x = pack16x2(tc[k], tc[k + 1], f16);
-    w.y = pack16x2(tc[k + 2], tc[k + 3], f16);
-    w.z = pack16x2(tc[k + 4], tc[k + 5], f16);
-    w.w = pack16x2(tc[k + 6], tc[k + 7], f16);
-    *reinterpret_cast<uint4*>(dst + k) = w;
+    for (int k = 0; k < 32; k += 2) *reinterpret_cast<uint32_t*>(dst + k) = pack16x2(tc[k], tc[k + 1], f16);
+  } else {
+    dst[0] = to16(tc[0], f16);
+#pragma unroll
+    for (int k = 1; k < 31; k += 2) *reinterpret_cast<uint32_t*>(dst + k) = pack16x2(tc[k], tc[k + 1], f16);
+    dst[31] = to16(tc[31], f16);
   }
-#pragma unroll
-  for (int k = H + 8 * NCH; k < 32; ++k) dst[k] = to16(tc[k], f16);
 }
 
 // V columns of a QKV projection with 16-bit (bf16 or fp16) storage, stored transposed per head
@@ -214,18 +215,7 @@ BAG_DEV void store_vt_warp(const Epi& e, int row, int col, float* v, float* sbuf
   uint16_t* vbase = reinterpret_cast<uint16_t*>(e.v);
   uint16_t* dst = vbase + (br1 ? e.br_vt : 0) + (long)cc * e.vpad + jr0;
   if (row0 + 31 < e.M && one_branch) {
-    // dst is 16-byte aligned exactly when jr0 is a multiple of 8 (vpad and the branch
-    // offset are multiples of 8 elements)
-    switch (jr0 & 7) {
-      case 0: store_vt_run<0>(dst, tc, f16); break;
-      case 1: store_vt_run<1>(dst, tc, f16); break;
-      case 2: store_vt_run<2>(dst, tc, f16); break;
-      case 3: store_vt_run<3>(dst, tc, f16); break;
-      case 4: store_vt_run<4>(dst, tc, f16); break;
-      case 5: store_vt_run<5>(dst, tc, f16); break;
-      case 6: store_vt_run<6>(dst, tc, f16); break;
-      default: store_vt_run<7>(dst, tc, f16); break;
-    }
+    store_vt_run(dst, tc, f16);
   } else {
 #pragma unroll
     for (int k = 0; k < 32; ++k) {
