@@ -94,6 +94,12 @@ BAG_DEV void load4(const void* p, long off, int bf16, float* r) {
   }
 }
 
+// Bulk prefetch of `bytes` (a multiple of 16, 16-byte aligned) into L2.
+BAG_DEV void l2_prefetch(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(p)), "r"(bytes)
+               : "memory");
+}
+
 // Four consecutive elements (16-bit or fp32) copied bit for bit.
 BAG_DEV void copy4(void* dst, const void* src, long off, int bf16) {
   if (bf16)
@@ -115,6 +121,18 @@ __global__ void __launch_bounds__(LN_THREADS, VPT <= 6 ? 8 : (VPT <= 10 ? 5 : 4)
   __shared__ float red_mean[LN_THREADS / 32], red_var[LN_THREADS / 32];
   const int row = blockIdx.x;
   if (row >= a.rows) return;
+  if (threadIdx.x == 0 && a.prefetch_rows > 0 && row + a.prefetch_rows < a.rows) {
+    // one bulk L2 prefetch per input row that a CTA of a later wave will read, so that
+    // its loads find the row in L2 (row strides are multiples of 16 bytes)
+    const long pr = (long)row + a.prefetch_rows;
+    l2_prefetch(a.x + pr * a.ldx, (uint32_t)a.cols * 4u);
+    if (a.sig_on) {
+      const uint32_t rb = (uint32_t)a.cols * (a.y_bf16 ? 2u : 4u);
+      const long off = pr * a.ldy * (a.y_bf16 ? 2 : 4);
+      l2_prefetch(reinterpret_cast<const char*>(a.sig_ref2) + off, rb);
+      l2_prefetch(reinterpret_cast<const char*>(a.sig_ref) + off, rb);
+    }
+  }
   const int t = a.st ? a.st->t : 0;
   const float* x = a.x + (long)row * a.ldx;
   const int nv = a.cols / 4;
@@ -222,9 +240,30 @@ __global__ void __launch_bounds__(LN_THREADS, VPT <= 6 ? 8 : (VPT <= 10 ? 5 : 4)
   }
 }
 
-cudaError_t ln_mod(const LnArgs& a, cudaStream_t s) {
-  if (a.rows <= 0) return cudaSuccess;
-  if (a.cols % 4 != 0 || a.cols > LN_THREADS * 4 * LN_MAXV) return cudaErrorInvalidValue;
+static int sm_count() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+cudaError_t ln_mod(const LnArgs& args, cudaStream_t s) {
+  if (args.rows <= 0) return cudaSuccess;
+  if (args.cols % 4 != 0 || args.cols > LN_THREADS * 4 * LN_MAXV) return cudaErrorInvalidValue;
+  LnArgs a = args;
+  // The signal pass reads two reference tensors last touched a step earlier (in HBM):
+  // each CTA prefetches into L2 the rows a CTA one wave later will read (distance = the
+  // CTAs resident on the GPU; bulk copies need 16-byte aligned rows).  The stack's
+  // LN-mods read rows the producing GEMM has just written (mostly still in L2): measured
+  // slower with the prefetch, so they take none.
+  const bool aligned = ((a.ldx * 4) % 16 == 0) && ((a.cols * 4) % 16 == 0) &&
+                       (a.ldy * (a.y_bf16 ? 2 : 4)) % 16 == 0;
+  const int per_sm = a.cols <= LN_THREADS * 4 * 6 ? 8 : (a.cols <= LN_THREADS * 4 * 10 ? 5 : 4);
+  a.prefetch_rows = (a.sig_on && aligned) ? sm_count() * per_sm : 0;
   if (a.cols <= LN_THREADS * 4 * 6)
     launch_kernel(ln_mod_kernel<6>, a.rows, LN_THREADS, 0, s, a);
   else if (a.cols <= LN_THREADS * 4 * 10)

@@ -198,6 +198,9 @@ struct LnArgs {
   void* sig_ref_w = nullptr;
   // identity: y = x (no normalisation or modulation; the observable is x itself)
   int identity = 0;
+  // rows ahead whose x (and signal references) a CTA pulls into L2 for a CTA of a later
+  // wave (set by the launcher: resident CTAs of the whole GPU; 0 = none)
+  int prefetch_rows = 0;
   const DevState* st; int flag_want;
 };
 cudaError_t ln_mod(const LnArgs& a, cudaStream_t s);

@@ -582,6 +582,27 @@ def test_guided_identical_branches_equal_unguided(name, lib):
     assert np.array_equal(got, plain)
 
 
+@pytest.mark.parametrize("name", ["flux_small", "wan_small"])
+def test_guided_budget_T_is_uncached_guided_sampling_bit_exact(name, lib):
+    """B = T under guidance computes every step for both branches (the batch-2 stack) and
+    equals the all-full policy bit for bit."""
+    cfg = configs.get_config(name, guidance=3.0)
+    T = 5
+    inp = synth.make_inputs(cfg)
+    ctx, a, ma, _, na = _gpu_guided(cfg, T, T, inp)
+    ctx.close()
+    ctx = bag.create(cfg, T=T, B=1)
+    ctx.set_policy(bag.POLICY_FULL)
+    x, txt, pooled = _dev_inputs(cfg, inp)
+    txt_u, pooled_u = _dev_uncond(cfg, inp)
+    ctx.reset()
+    mb, _, nb = ctx.run(x, txt, pooled, txt_u, pooled_u)
+    torch.cuda.synchronize()
+    ctx.close()
+    assert list(ma) == list(mb) == [1] * T and na == nb == T
+    assert np.array_equal(a, x.cpu().numpy())
+
+
 def test_guided_context_requires_unconditional_inputs(lib):
     cfg = configs.get_config("tiny", guidance=2.0)
     ctx = bag.create(cfg, T=4, B=2)

@@ -33,7 +33,15 @@ CASES = [
     ("qwen_wide", {}, None),
     ("wan_wide", {}, None),
     ("flux_wide", dict(qk_norm=True), 4.0),
+    ("wan_wide", {}, 5.0),
+    ("qwen_wide", dict(observable="embedded"), 4.0),
 ]
+# Cases where the operand precision itself exceeds the stated 2e-2 bar: under guidance
+# the velocity is v_u + g (v_c - v_u), which multiplies the branches' errors by about
+# sqrt((g - 1)^2 + g^2); at Wan width and g = 5 the error model alone reaches a max-abs
+# of 2.8e-2 x RMS.  There the GPU is held to the model instead (max-abs and RMS within
+# 1.25x of the model's).
+PRECISION_BOUND = {("wan_wide", 5.0)}
 
 
 def _dev(cfg, a):
@@ -49,7 +57,8 @@ def _cond(cfg, inp, guided):
 
 
 @pytest.mark.parametrize("name,over,guidance", CASES,
-                         ids=["flux", "qwen", "wan-unipc", "flux-guided-qknorm"])
+                         ids=["flux", "qwen", "wan-unipc", "flux-guided-qknorm", "wan-unipc-guided",
+                              "qwen-guided-embedded-observable"])
 def test_wide_sample_parity(name, over, guidance, lib):
     if guidance is not None:
         over = dict(over, guidance=guidance)
@@ -95,7 +104,10 @@ def test_wide_sample_parity(name, over, guidance, lib):
     print(f"{name} {over}: max|err| = {err:.4e} = {err / rms:.3e} x RMS {rms:.4f} (model "
           f"{np.max(np.abs(model['x'] - ref['x'])) / rms:.3e}); RMS(err) = {rms_err / rms:.3e} x RMS "
           f"(model {rms_model / rms:.3e})")
-    assert err <= TOL_BF16 * rms, (err, rms)
+    if (name, guidance) in PRECISION_BOUND:
+        assert err <= 1.25 * float(np.max(np.abs(model["x"] - ref["x"]))), (err, rms)
+    else:
+        assert err <= TOL_BF16 * rms, (err, rms)
     assert rms_err <= 1.25 * rms_model, (rms_err, rms_model)
     # the stack moved the latent well beyond the error (not a near-identity network)
     assert float(np.max(np.abs(ref["x"] - inp["x"]))) > 20 * err
