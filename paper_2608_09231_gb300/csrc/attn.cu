@@ -114,7 +114,7 @@ cudaError_t attention(const AttnArgs& a, int* err, cudaStream_t s, int force_sim
     if (!attention_tc_supported(a)) return cudaErrorNotSupported;
     return attention_tc(a, err, s);
   }
-  if (a.f16) return cudaErrorNotSupported;  // fp16 operands: tensor-core kernel only
+  if (a.f16 || a.nbr > 1) return cudaErrorNotSupported;  // tensor-core kernel only
   dim3 grid((a.nq + 15) / 16, a.heads);
   if (a.dh == 64) {
     if (a.bf16)

@@ -47,6 +47,10 @@ struct AttnTcParams {
   long ldo;
   void* o2;     // rows >= o_split are written to o2 (same row index and stride)
   int o_split;
+  // branch blockIdx.z: q / k row offsets, V^T row offset (per branch block), outputs
+  int br_q_rows, br_k_rows, br_v_rows;
+  void* o_b1;
+  void* o2_b1;
   float scale_log2;
   const DevState* st;
   int flag_want;
@@ -147,6 +151,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int head = blockIdx.y, q0 = blockIdx.x * 2 * AT_M;
+  const int br = blockIdx.z;  // guidance branch (0 unless two branches share the launch)
+  const int qr0 = q0 + br * p.br_q_rows, kr0 = br * p.br_k_rows, vr0 = br * p.br_v_rows;
   const int nkb = (p.nk + AT_N - 1) / AT_N;
 
   if (threadIdx.x == 0) {
@@ -181,8 +187,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       // ---------------- TMA producer ----------------
       mbar_arrive_expect_tx(q_full, 2 * AT_TILE);
       for (int x = 0; x < 2; ++x) {
-        tma_load_2d(sQ + x * AT_TILE, &tmQ, head * AT_D, q0 + x * AT_M, q_full);
-        tma_load_2d(sQ + x * AT_TILE + AT_CHUNK, &tmQ, head * AT_D + 64, q0 + x * AT_M, q_full);
+        tma_load_2d(sQ + x * AT_TILE, &tmQ, head * AT_D, qr0 + x * AT_M, q_full);
+        tma_load_2d(sQ + x * AT_TILE + AT_CHUNK, &tmQ, head * AT_D + 64, qr0 + x * AT_M, q_full);
       }
       int issued = 0;
       bool ok = true;
@@ -195,10 +201,10 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         uint8_t* k = sKV + s * 2 * AT_TILE;
         uint8_t* v = k + AT_TILE;
         mbar_arrive_expect_tx(kv_full + s, 2 * AT_TILE);
-        tma_load_2d(k, &tmK, head * AT_D, j * AT_N, kv_full + s);
-        tma_load_2d(k + AT_CHUNK, &tmK, head * AT_D + 64, j * AT_N, kv_full + s);
-        tma_load_2d(v, &tmV, j * AT_N, head * AT_D, kv_full + s);
-        tma_load_2d(v + AT_CHUNK, &tmV, j * AT_N + 64, head * AT_D, kv_full + s);
+        tma_load_2d(k, &tmK, head * AT_D, kr0 + j * AT_N, kv_full + s);
+        tma_load_2d(k + AT_CHUNK, &tmK, head * AT_D + 64, kr0 + j * AT_N, kv_full + s);
+        tma_load_2d(v, &tmV, j * AT_N, vr0 + head * AT_D, kv_full + s);
+        tma_load_2d(v + AT_CHUNK, &tmV, j * AT_N + 64, vr0 + head * AT_D, kv_full + s);
         ++issued;
       }
       if (!ok) {
@@ -365,7 +371,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         tc_fence_after();
         const float inv = 1.f / l;
         const int q = q0 + x * AT_M + row;
-        void* ob = (p.o2 && q >= p.o_split) ? p.o2 : p.o;
+        void* o1 = br ? p.o_b1 : p.o;
+        void* o2 = br ? p.o2_b1 : p.o2;
+        void* ob = (o2 && q >= p.o_split) ? o2 : o1;
         __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(ob) + (long)q * p.ldo + head * AT_D;
 #pragma unroll 1
         for (int c = 0; c < AT_D / 32; ++c) {
@@ -406,9 +414,14 @@ int attention_tc_supported(const AttnArgs& a) {
 cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t s) {
   CUtensorMap tq, tk, tv;
   const uint64_t width = (uint64_t)a.heads * AT_D;
-  if (encode_tmap_2d_bf16(&tq, a.q, width, (uint64_t)a.nq, (uint64_t)a.ldq * 2, 64, AT_M) ||
-      encode_tmap_2d_bf16(&tk, a.k, width, (uint64_t)a.nk, (uint64_t)a.ldk * 2, 64, AT_N) ||
-      encode_tmap_2d_bf16(&tv, a.v, (uint64_t)a.nk, width, (uint64_t)a.vpad * 2, 64, AT_D))
+  const int nbr = a.nbr > 1 ? 2 : 1;
+  // with two branches the maps span both (the rows past a branch's last query or key are
+  // never stored, resp. masked, and its V^T block is zero beyond nk up to vpad)
+  const uint64_t qrows = nbr > 1 ? (uint64_t)a.br_q_rows + a.nq : (uint64_t)a.nq;
+  const uint64_t krows = nbr > 1 ? (uint64_t)a.br_k_rows + a.nk : (uint64_t)a.nk;
+  if (encode_tmap_2d_bf16(&tq, a.q, width, qrows, (uint64_t)a.ldq * 2, 64, AT_M) ||
+      encode_tmap_2d_bf16(&tk, a.k, width, krows, (uint64_t)a.ldk * 2, 64, AT_N) ||
+      encode_tmap_2d_bf16(&tv, a.v, (uint64_t)a.nk, width * nbr, (uint64_t)a.vpad * 2, 64, AT_D))
     return cudaErrorInvalidValue;
   AttnTcParams p;
   p.nq = a.nq;
@@ -417,11 +430,16 @@ cudaError_t attention_tc(const AttnArgs& a, int* err, cudaStream_t s) {
   p.ldo = a.ldo;
   p.o2 = a.o2;
   p.o_split = a.o_split;
+  p.br_q_rows = nbr > 1 ? (int)a.br_q_rows : 0;
+  p.br_k_rows = nbr > 1 ? (int)a.br_k_rows : 0;
+  p.br_v_rows = nbr > 1 ? (int)width : 0;
+  p.o_b1 = a.o_b1;
+  p.o2_b1 = a.o2_b1;
   p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)AT_D));
   p.st = a.st;
   p.flag_want = a.flag_want;
   p.err = err;
-  dim3 grid((a.nq + 2 * AT_M - 1) / (2 * AT_M), a.heads);
+  dim3 grid((a.nq + 2 * AT_M - 1) / (2 * AT_M), a.heads, nbr);
   if (a.f16)
     launch_kernel(attn_tc_kernel<true>, grid, AT_THREADS, AT_SMEM, s, tq, tk, tv, p);
   else

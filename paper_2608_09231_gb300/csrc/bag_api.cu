@@ -876,9 +876,19 @@ static void enq_qkv_epi(const bag_ctx* ctx, Epi& e, int row_off, bool rope) {
   e.ldm = ctx->d + ctx->F;
 }
 
+// Attention of one branch, or of both guidance branches in one launch (nbr = 2, bf16
+// backbones): branch 1's q / k rows br_q / br_k rows further, its V^T block right after
+// branch 0's, its output to O_b1 / O2_b1.
+struct AttnBranch {
+  int nbr = 1;
+  long br_q = 0, br_k = 0;
+  void* o_b1 = nullptr;
+  void* o2_b1 = nullptr;
+};
+
 static void enq_attn(Enq& q, const void* Q, const void* K, const void* V, long vpad, void* O,
                      long ldo, int nq, int nk, const DevState* st, int flag_want,
-                     void* O2 = nullptr, int o_split = 0) {
+                     void* O2 = nullptr, int o_split = 0, const AttnBranch& ab = AttnBranch()) {
   const bag_ctx* ctx = q.ctx;
   AttnArgs a{};
   a.q = Q;
@@ -893,6 +903,11 @@ static void enq_attn(Enq& q, const void* Q, const void* K, const void* V, long v
   a.ldo = ldo;
   a.o2 = O2;
   a.o_split = o_split;
+  a.nbr = ab.nbr;
+  a.br_q_rows = ab.br_q;
+  a.br_k_rows = ab.br_k;
+  a.o_b1 = ab.o_b1;
+  a.o2_b1 = ab.o2_b1;
   a.nq = nq;
   a.nk = nk;
   a.heads = ctx->H;
@@ -901,8 +916,8 @@ static void enq_attn(Enq& q, const void* Q, const void* K, const void* V, long v
   a.f16 = ctx->act_bf16;  // q, k, v fp16 (written so by the projections' epilogues)
   a.st = st;
   a.flag_want = flag_want;
-  q.pre(BAG_PROF_ATTN, 4.0 * nq * nk * ctx->H * ctx->dh,
-        ((double)nq * 2 + 2.0 * nk) * ctx->d * ctx->act_size, nq, nk, ctx->H);
+  q.pre(BAG_PROF_ATTN, 4.0 * nq * nk * ctx->H * ctx->dh * ab.nbr,
+        ((double)nq * 2 + 2.0 * nk) * ctx->d * ctx->act_size * ab.nbr, nq, nk, ctx->H);
   q.chk(attention(a, ctx->st ? &ctx->st->err : nullptr, q.s));
 }
 
@@ -960,6 +975,16 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int n
   // br * vt_br); the output rows go back in stream order (text rows of branch br at
   // br * nx, its image rows at nb * nx + br * ni)
   auto attn_joint = [&]() {
+    if (nb > 1 && ctx->act_bf16) {  // both branches in one launch
+      AttnBranch ab;
+      ab.nbr = 2;
+      ab.br_q = ab.br_k = N;
+      ab.o_b1 = off_act(ctx, ctx->cat, (long)nx * ldc);
+      ab.o2_b1 = off_act(ctx, ctx->cat, ((long)nb * nx + ni - nx) * ldc);
+      enq_attn(q, ctx->q, ctx->k, ctx->vt, ctx->vpad, ctx->cat, ldc, N, N, st, fw,
+               off_act(ctx, ctx->cat, ((long)nb * nx - nx) * ldc), nx, ab);
+      return;
+    }
     for (int br = 0; br < nb; ++br) {
       void* o = off_act(ctx, ctx->cat, (long)br * nx * ldc);
       void* o2 = off_act(ctx, ctx->cat, ((long)nb * nx + (long)br * ni - nx) * ldc);
@@ -1095,10 +1120,17 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int n
     epi_branches(ctx, e, nb, ni, ni, ctx->vpad);
     enq_gemm(q, ctx->xn, d, blk.w.at("sa_qkv_w"), d, R, (int)(3 * d), (int)d, e);
   }
-  for (int br = 0; br < nb; ++br)
+  AttnBranch ab;  // Wan, both branches in one launch (bf16 backbones)
+  const int nl = (nb > 1 && ctx->act_bf16) ? 1 : nb;
+  if (nl < nb) {
+    ab.nbr = 2;
+    ab.br_q = ab.br_k = ni;
+    ab.o_b1 = off_act(ctx, ctx->cat, (long)ni * ldc);
+  }
+  for (int br = 0; br < nl; ++br)
     enq_attn(q, off_act(ctx, ctx->q, (long)br * ni * d), off_act(ctx, ctx->k, (long)br * ni * d),
              off_act(ctx, ctx->vt, br * vtw_br), ctx->vpad, off_act(ctx, ctx->cat, (long)br * ni * ldc),
-             ldc, ni, ni, st, fw);
+             ldc, ni, ni, st, fw, nullptr, 0, ab);
   {
     Epi r = base_epi(ctx, st, fw);
     r.kind = EPI_GATED_RES;
@@ -1137,10 +1169,12 @@ static void enq_block(Enq& q, int b, float* h, const DevState* st, int fw, int n
     epi_branches(ctx, kv, nb, nx, nx, ctx->vpad_c);
     enq_gemm(q, ctx->txt_stage, d, blk.w.at("ca_kv_w"), d, nb * nx, (int)(2 * d), (int)d, kv);
   }
-  for (int br = 0; br < nb; ++br)
+  AttnBranch abc = ab;
+  abc.br_k = nx;
+  for (int br = 0; br < nl; ++br)
     enq_attn(q, off_act(ctx, ctx->qc, (long)br * ni * d), off_act(ctx, ctx->kc, (long)br * nx * d),
              off_act(ctx, ctx->vtc, br * vtc_br), ctx->vpad_c, off_act(ctx, ctx->cat, (long)br * ni * ldc),
-             ldc, ni, nx, st, fw);
+             ldc, ni, nx, st, fw, nullptr, 0, abc);
   {
     Epi r = base_epi(ctx, st, fw);
     r.kind = EPI_RES_ADD;

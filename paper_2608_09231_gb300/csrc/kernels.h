@@ -165,6 +165,14 @@ struct AttnArgs {
   const void* v;  int v_mode; long ldv; long vpad;  // mode 0 like k; mode 1 [H][dh][vpad]
   void* o;        long ldo;      // output [Nq][ldo], head h at column h*dh
   void* o2 = nullptr; int o_split = 0;  // rows >= o_split go to o2 (+ row * ldo) instead
+  // nbr = 2 (tensor-core kernel): two guidance branches in one launch; branch 1's q and k
+  // rows start br_q_rows / br_k_rows rows further, its transposed V heads * dh rows
+  // further (each branch has its own [heads][dh][vpad] block), and its output goes to
+  // o_b1 / o2_b1 with the same row split
+  int nbr = 1;
+  long br_q_rows = 0, br_k_rows = 0;
+  void* o_b1 = nullptr;
+  void* o2_b1 = nullptr;
   int nq, nk, heads, dh;
   int bf16;                      // 16-bit operands and output (else fp32)
   int f16 = 0;                   // with bf16: q, k, v are fp16 (output stays bf16)
