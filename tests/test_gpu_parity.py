@@ -603,6 +603,29 @@ def test_guided_budget_T_is_uncached_guided_sampling_bit_exact(name, lib):
     assert np.array_equal(a, x.cpu().numpy())
 
 
+@pytest.mark.parametrize("name", ["flux_small", "wan_small"])
+def test_guided_step_api_matches_run(name, lib):
+    """bag_step under guidance (the batch-2 stack, one shared mask) reproduces bag_run bit
+    for bit, step by step."""
+    cfg = configs.get_config(name, guidance=2.5)
+    T, B = 6, 3
+    ctx = bag.create(cfg, T=T, B=B)
+    inp = synth.make_inputs(cfg)
+    x, txt, pooled = _dev_inputs(cfg, inp)
+    txt_u, pooled_u = _dev_uncond(cfg, inp)
+    x0 = x.clone()
+    m_run, _, _ = ctx.run(x, txt, pooled, txt_u, pooled_u)
+    ctx.reset()
+    xs = x0.clone()
+    flags = torch.zeros(T, dtype=torch.int32, device="cuda")
+    for t in range(T):
+        ctx.step(xs, t, txt, pooled, xs, flags[t:], txt_u, pooled_u)
+    torch.cuda.synchronize()
+    ctx.close()
+    assert list(flags.cpu().numpy()) == list(m_run) and int(flags.sum()) == B
+    assert torch.equal(xs, x)
+
+
 def test_guided_context_requires_unconditional_inputs(lib):
     cfg = configs.get_config("tiny", guidance=2.0)
     ctx = bag.create(cfg, T=4, B=2)
