@@ -383,6 +383,34 @@ def job_seconds_per_sample(ms_per_step_max, world):
     return ms_per_step_max / 1e3 / world
 
 
+def budget_overhead(sweep, prof, T):
+    """How s/sample scales with the budget (the benchmark spec: with B/T plus a measured gate and
+    skip overhead).  sweep: {B: s/sample}; prof: the profiled sample's per-class times.
+    A least-squares line s(B) = slope * B + fixed over the swept budgets gives the cost of
+    one more full step and the budget-independent part; the profiled sample gives the
+    per-step cost of the method's own kernels (signal, gate, cache refresh / reuse)."""
+    out = {}
+    pts = sorted((int(b), float(v)) for b, v in sweep.items())
+    if len(pts) >= 2:
+        n = len(pts)
+        mb = sum(b for b, _ in pts) / n
+        mv = sum(v for _, v in pts) / n
+        sxx = sum((b - mb) ** 2 for b, _ in pts)
+        slope = sum((b - mb) * (v - mv) for b, v in pts) / sxx
+        out["fit_ms_per_full_step"] = slope * 1e3
+        out["fit_fixed_ms"] = (mv - slope * mb) * 1e3
+        out["fit_max_residual_ms"] = max(abs(v - (mv + slope * (b - mb))) for b, v in pts) * 1e3
+    total = sum(v["ms"] for v in prof.values())
+    own = 0.0
+    for k in ("signal", "gate", "cache"):
+        if k in prof:
+            out[f"{k}_us_per_step"] = prof[k]["ms"] * 1e3 / T
+            own += prof[k]["ms"]
+    if total > 0:
+        out["method_kernels_share"] = own / total
+    return out
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -609,6 +637,7 @@ def main():
                                      "attention": attn_tflops, "peak": peak_t,
                                      "frac": block_tflops / peak_t},
                 "kernels": kernels, "budget_sweep_s_per_sample": sweep,
+                "overhead": budget_overhead(sweep, prof, T),
                 "cpu_baseline": cpu}
         print(json.dumps(line))
     ctx.close()

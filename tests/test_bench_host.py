@@ -71,3 +71,17 @@ def test_job_throughput_counts_every_replica(bench):
     # N replicas finish N samples in the slowest replica's step time
     assert bench.job_seconds_per_sample(1000.0, 1) == 1.0
     assert bench.job_seconds_per_sample(1000.0, 4) == 0.25
+
+
+def test_budget_overhead_fit(bench):
+    """The budget fit recovers an exact line s(B) = 0.05 B + 0.02 and the per-step cost of
+    the method's own kernels from the profiled classes."""
+    sweep = {str(b): 0.05 * b + 0.02 for b in (25, 20, 15, 10)}
+    prof = {"gemm": {"ms": 900.0}, "attention": {"ms": 80.0}, "signal": {"ms": 2.0},
+            "gate": {"ms": 1.0}, "cache": {"ms": 1.5}, "norm": {"ms": 15.5}}
+    o = bench.budget_overhead(sweep, prof, 50)
+    assert abs(o["fit_ms_per_full_step"] - 50.0) < 1e-9
+    assert abs(o["fit_fixed_ms"] - 20.0) < 1e-9 and o["fit_max_residual_ms"] < 1e-9
+    assert abs(o["signal_us_per_step"] - 40.0) < 1e-9 and abs(o["gate_us_per_step"] - 20.0) < 1e-9
+    assert abs(o["method_kernels_share"] - 4.5 / 1000.0) < 1e-12
+    assert "fit_ms_per_full_step" not in bench.budget_overhead({"20": 1.0}, prof, 50)
